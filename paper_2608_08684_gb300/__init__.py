@@ -1,0 +1,10 @@
+"""RippleKV serving hot path on GB300 (sm_103a).
+
+Submodules:
+  ripple  -- ctypes binding of the C-ABI library libripple.so (the product path)
+  synth   -- seeded synthetic inputs (no step of the method)
+  build   -- in-tree build of libripple.so with nvcc/gcc
+  replica -- host logic of independent multi-GPU replicas
+
+Nothing is imported eagerly, so that importing the package never loads CUDA.
+"""
