@@ -1,0 +1,544 @@
+#!/usr/bin/env python3
+"""Benchmark of the RippleKV serving hot path on GB300.
+
+One step = the whole path on one synthetic batch: host budget allocation
+(Eqs. 9-12), compression of every layer (scoring, pooling, top-k, gather) and
+the workload's decode steps over the ragged caches, all through the C ABI.
+
+Default workload: the Llama-3-8B-shaped 32k stack (32 layers, 32 q / 8 KV
+heads, d = 128, batch 4, T = 32768, bf16, average budget 1024, ratio 8, 128
+decode steps). Inputs are synthetic (seeded), generated on the device and
+resident in HBM when the timed region starts; per layer K + V is 537 MB, far
+above the 129 MB L2, so no flush is needed between steps.
+
+Output: one JSON line (rank 0). `value` = prompt tokens compressed and then
+decoded per second over whole steps (B * T * ranks / step time). Extra keys
+break the step down: compression-only tokens/s and decode-attention GB/s, each
+against the measured HBM copy bandwidth.
+
+--impl reference times the CPU oracle (the test-infrastructure restatement of
+the paper) on a bounded sample of the same workload, extrapolated to a step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+HBM_FALLBACK_GBS = 6800.0
+REASON_BITS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+               0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+               0x100: "display_clock_setting"}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="llama8b-32k")
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target CPU seconds of the oracle sample")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_FALLBACK_GBS, "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    def __init__(self, gpu_index: int):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active")
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(self.gpu_index)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons, power = [], None, set(), []
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 5:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+                power.append(float(parts[3]))
+                bits = int(parts[4], 16)
+            except ValueError:
+                continue
+            for b, name in REASON_BITS.items():
+                if bits & b and name != "gpu_idle":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# ----------------------------------------------------------------- workload state
+
+
+class Serving:
+    """Device-resident inputs, outputs and workspaces of one workload."""
+
+    def __init__(self, R, synth, wl, device):
+        import torch
+        self.R, self.wl, self.dev = R, wl, device
+        L, B, Hq, Hkv, d = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+        self.sens = synth.sensitivity_profile(wl)
+        self.budgets = R.ripple_alloc_budgets(self.sens, wl.ratio, wl.gamma, wl.global_budget)
+        self.n_keep = [R.ripple_keep_count(b, wl.seq_len, wl.window) for b in self.budgets]
+        self.caps = [n + wl.decode_steps for n in self.n_keep]
+        self.q_win, self.k, self.v = [], [], []
+        for layer in range(L):
+            self.q_win.append(synth.layer_window_queries(wl, layer, device))
+            self.k.append(synth.layer_keys(wl, layer, device))
+            self.v.append(synth.layer_values(wl, layer, device))
+        self.desc = R.layer_desc(B, Hq, Hkv, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                                 wl.torch_dtype)
+        self.ws = torch.empty(R.ripple_compress_workspace_bytes(self.desc), dtype=torch.uint8,
+                              device=device)
+        self.k_out = [torch.zeros(B, Hkv, c, d, dtype=wl.torch_dtype, device=device)
+                      for c in self.caps]
+        self.v_out = [torch.zeros_like(t) for t in self.k_out]
+        self.idx = [torch.empty(B * Hkv * n, dtype=torch.int32, device=device)
+                    for n in self.n_keep]
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+        self.dq, self.dk, self.dv = [], [], []
+        for t in range(wl.decode_steps):
+            q, kn, vn = synth.decode_inputs(wl, t, device)
+            self.dq.append(q)
+            self.dk.append(kn)
+            self.dv.append(vn)
+        self.ddesc = R.decode_desc(L, B, Hq, Hkv, d, wl.torch_dtype)
+        self.tables = R.DecodeTables(self.k_out, self.v_out)
+        self.dws = torch.empty(R.ripple_decode_workspace_bytes(self.ddesc, self.caps),
+                               dtype=torch.uint8, device=device)
+        self.lens0 = torch.tensor(self.n_keep, dtype=torch.int32, device=device)
+        self.lens = self.lens0.clone()
+        self.out = torch.empty(wl.decode_steps, L, B, Hq, d, dtype=torch.float32, device=device)
+
+    def step(self, timers=None):
+        """One pass of the whole path; timers = (compress_events, decode_events) or None."""
+        import torch
+        R, wl = self.R, self.wl
+        budgets = R.ripple_alloc_budgets(self.sens, wl.ratio, wl.gamma, wl.global_budget)
+        assert budgets == self.budgets
+        ev = (lambda: torch.cuda.Event(enable_timing=True)) if timers else None
+        if timers:
+            c0 = ev()
+            c0.record()
+        for layer in range(wl.n_layers):
+            n = R.ripple_compress_layer(self.desc, budgets[layer], self.q_win[layer], self.k[layer],
+                                        self.v[layer], self.k_out[layer], self.v_out[layer],
+                                        self.idx[layer], self.ws, dev_status=self.status)
+            assert n == self.n_keep[layer]
+        if timers:
+            c1 = ev()
+            c1.record()
+            timers[0].append((c0, c1))
+        self.lens.copy_(self.lens0)
+        for t in range(wl.decode_steps):
+            if timers:
+                d0 = ev()
+                d0.record()
+            R.ripple_decode_attn(self.ddesc, self.dq[t], self.dk[t], self.dv[t], self.tables,
+                                 self.lens, self.out[t], self.dws, dev_status=self.status)
+            if timers:
+                d1 = ev()
+                d1.record()
+                timers[1].append((d0, d1))
+
+    # algorithmic bytes (what the method must move)
+    def compress_bytes(self):
+        wl, e = self.wl, self.wl.elem_bytes
+        tot = 0
+        for n in self.n_keep:
+            tot += wl.batch * wl.n_kv_heads * wl.head_dim * e * (wl.seq_len + 3 * n)
+            tot += wl.batch * wl.n_q_heads * wl.window * wl.head_dim * e
+        return tot
+
+    def decode_bytes_per_step(self):
+        """Average over the decode steps: K/V rows read (retained + appended +
+        the new row), queries read, outputs written, new rows read and appended."""
+        wl, e = self.wl, self.wl.elem_bytes
+        L, B, Hq, Hkv, d = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+        tot = 0
+        for t in range(wl.decode_steps):
+            for n in self.n_keep:
+                tot += B * Hkv * (n + t + 1) * d * e * 2
+            tot += L * B * Hq * d * (e + 4) + L * B * Hkv * d * e * 4
+        return tot / wl.decode_steps
+
+
+def elapsed_ms(pairs):
+    return [a.elapsed_time(b) for a, b in pairs]
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_08684_gb300 import build as _build
+    from paper_2608_08684_gb300 import synth
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=device)
+    if rank == 0:
+        _build.build_library()
+    if world > 1:
+        dist.barrier()
+    from paper_2608_08684_gb300 import ripple as R
+
+    wl = synth.WORKLOADS[args.workload]
+    # independent replicas: every rank serves its own batch (weak scaling)
+    wl = wl.replace(seed=wl.seed + 1000 * rank) if rank else wl
+    st = Serving(R, synth, wl, device)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        st.step()
+    barrier()
+    assert int(st.status.item()) == 0, f"device status {int(st.status.item())}"
+    launches0 = R.ripple_kernel_launches()
+    timers = ([], [])
+    gpu_index = int(os.environ.get("CUDA_VISIBLE_DEVICES", str(local_rank)).split(",")[0]) \
+        if os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",")[0].isdigit() else local_rank
+    with ClockSampler(gpu_index) as clocks:
+        barrier()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(args.steps):
+            st.step(timers)
+        t1.record()
+        barrier()
+    launches = R.ripple_kernel_launches() - launches0
+    assert int(st.status.item()) == 0
+    total_ms = t0.elapsed_time(t1)
+    if world > 1:
+        tt = torch.tensor([total_ms], device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    tokens = wl.batch * wl.seq_len * world
+    value = tokens / (ms_per_step / 1e3)
+
+    comp_ms = elapsed_ms(timers[0])
+    dec_ms = elapsed_ms(timers[1])
+    hbm, hbm_src = measured_peaks()
+    comp_avg = statistics.mean(comp_ms)
+    dec_avg = statistics.mean(dec_ms)
+    comp_gbs = st.compress_bytes() / (comp_avg / 1e3) / 1e9
+    dec_gbs = st.decode_bytes_per_step() / (dec_avg / 1e3) / 1e9
+    comp_total = comp_avg
+    dec_total = dec_avg * wl.decode_steps
+    roof_dec = {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(dec_gbs / hbm, 4), "traffic": None,
+                "kernel": "ripple_decode_attn (decode_partial + decode_combine)",
+                "bytes_per_launch": round(st.decode_bytes_per_step()),
+                "ms_per_launch": round(dec_avg, 5), "peak_source": hbm_src}
+    roof_comp = {"bound": "hbm", "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s",
+                 "frac": round(comp_gbs / hbm, 4), "traffic": None,
+                 "kernel": "ripple_compress_layer x all layers",
+                 "bytes_per_launch": round(st.compress_bytes()),
+                 "ms_per_launch": round(comp_avg, 4), "peak_source": hbm_src}
+    dominant = roof_dec if dec_total >= comp_total else roof_comp
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = measure_e2e(st, args, torch, tokens // world * world)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(st, args.cpu_seconds)
+    if rank != 0:
+        return
+    line = {
+        "metric": "compressed-prefill tokens/s; ragged decode-attn HBM GB/s vs GB300 peak",
+        "value": round(value, 1), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch,
+                   "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+                   "seq_len": wl.seq_len, "window": wl.window, "pool_kernel": wl.pool_kernel,
+                   "ratio": wl.ratio, "avg_budget": wl.avg_budget,
+                   "decode_steps": wl.decode_steps, "budgets": st.budgets,
+                   "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (K+V per layer %.0f MB), no flush"
+                         % (2 * wl.batch * wl.n_kv_heads * wl.seq_len * wl.head_dim
+                            * wl.elem_bytes / 1e6)},
+        "compress": {"tokens_per_s": round(tokens / world / (comp_avg / 1e3), 1),
+                     "ms": round(comp_avg, 4), "gbs": round(comp_gbs, 1),
+                     "frac_hbm": round(comp_gbs / hbm, 4),
+                     "frac_8tbs_spec": round(comp_gbs / 8000.0, 4)},
+        "decode_attn": {"gbs": round(dec_gbs, 1), "ms_per_step": round(dec_avg, 5),
+                        "frac_hbm": round(dec_gbs / hbm, 4),
+                        "frac_8tbs_spec": round(dec_gbs / 8000.0, 4)},
+        "roofline": dominant,
+        "roofline_compress": roof_comp,
+        "roofline_decode": roof_dec,
+        "gpu_launches": launches,
+        "clocks": clocks.summary(),
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if cpu:
+        line["cpu_baseline"] = cpu
+    print(json.dumps(line), flush=True)
+
+
+def measure_e2e(st, args, torch, tokens):
+    """Same metric through the C ABI from pinned host buffers: every step copies
+    the layer inputs and decode inputs host->device and reads the decode
+    outputs back, inside the timed region."""
+    wl = st.wl
+    pin = lambda t: t.to("cpu").pin_memory()
+    hq = [pin(t) for t in st.q_win]
+    hk = [pin(t) for t in st.k]
+    hv = [pin(t) for t in st.v]
+    hdq = [pin(t) for t in st.dq]
+    hdk = [pin(t) for t in st.dk]
+    hdv = [pin(t) for t in st.dv]
+    hout = torch.empty(st.out.shape, dtype=st.out.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv + hdq + hdk + hdv)
+    d2h = hout.numel() * hout.element_size()
+
+    def step():
+        for layer in range(wl.n_layers):
+            st.q_win[layer].copy_(hq[layer], non_blocking=True)
+            st.k[layer].copy_(hk[layer], non_blocking=True)
+            st.v[layer].copy_(hv[layer], non_blocking=True)
+        for t in range(wl.decode_steps):
+            st.dq[t].copy_(hdq[t], non_blocking=True)
+            st.dk[t].copy_(hdk[t], non_blocking=True)
+            st.dv[t].copy_(hdv[t], non_blocking=True)
+        st.step()
+        hout.copy_(st.out, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.e2e_steps):
+        step()
+    t1.record()
+    torch.cuda.synchronize()
+    ms = t0.elapsed_time(t1) / args.e2e_steps
+    return {"value": round(tokens / (ms / 1e3), 1), "unit": "tokens/s", "ms_per_step": round(ms, 3),
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+
+
+# ----------------------------------------------------------------- CPU oracle
+
+
+def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s):
+    """Times the oracle on a bounded sample of compression units and decode
+    groups and extrapolates to one full step. Returns (step seconds, sample text)."""
+    import numpy as np
+
+    from oracle import ripple_oracle as O
+    scale = 1.0 / math.sqrt(wl.head_dim)
+    units_total = wl.n_layers * wl.batch * wl.n_kv_heads
+    # compression sample: units of the largest-budget layer, round robin over (b, h)
+    layer = int(np.argmax(budgets))
+    t_comp, n_comp = 0.0, 0
+    while t_comp < 0.75 * target_s and n_comp < wl.batch * wl.n_kv_heads:
+        b, h = divmod(n_comp, wl.n_kv_heads)
+        q, k, v = get_unit(layer, b, h)
+        t = time.perf_counter()
+        O.compress_unit(q, k, v, budgets[layer], wl.window, scale, wl.pool_kernel)
+        t_comp += time.perf_counter() - t
+        n_comp += 1
+    # decode sample: one (layer, b, h) group per layer, over min(8, steps) steps
+    steps = min(8, wl.decode_steps)
+    t_dec, n_dec = 0.0, 0
+    for layer in range(wl.n_layers):
+        if t_dec > 0.25 * target_s:
+            break
+        kk, vv, qs, kns, vns = get_decode(layer, steps)
+        rows_k, rows_v = kk, vv
+        t = time.perf_counter()
+        for s in range(steps):
+            rows_k = np.vstack([rows_k, kns[s][None]])
+            rows_v = np.vstack([rows_v, vns[s][None]])
+            O.decode_attention(qs[s], rows_k, rows_v, scale)
+        t_dec += time.perf_counter() - t
+        n_dec += steps
+    per_unit = t_comp / n_comp
+    per_group_step = t_dec / n_dec
+    step_s = per_unit * units_total + per_group_step * (
+        wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps)
+    sample = (f"{n_comp} compression units of layer {layer} (T={wl.seq_len}) and {n_dec} "
+              f"decode (group, step) pairs; extrapolated to {units_total} units and "
+              f"{wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps} group-steps")
+    return step_s, sample, t_comp + t_dec
+
+
+def _threads():
+    try:
+        import threadpoolctl
+        info = threadpoolctl.threadpool_info()
+        n = max((i.get("num_threads", 1) for i in info), default=1)
+        return int(n)
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(st, target_s):
+    import numpy as np
+
+    from paper_2608_08684_gb300 import synth
+    wl = st.wl
+    G = wl.group
+
+    def get_unit(layer, b, h):
+        return (synth.to_f64(st.q_win[layer][b, h * G:(h + 1) * G]), synth.to_f64(st.k[layer][b, h]),
+                synth.to_f64(st.v[layer][b, h]))
+
+    def get_decode(layer, steps):
+        n = st.n_keep[layer]
+        idx = st.idx[layer].view(wl.batch, wl.n_kv_heads, n)[0, 0].long()
+        kk = synth.to_f64(st.k[layer][0, 0].index_select(0, idx))
+        vv = synth.to_f64(st.v[layer][0, 0].index_select(0, idx))
+        qs = [synth.to_f64(st.dq[s][layer, 0, 0:G]) for s in range(steps)]
+        kns = [synth.to_f64(st.dk[s][layer, 0, 0]) for s in range(steps)]
+        vns = [synth.to_f64(st.dv[s][layer, 0, 0]) for s in range(steps)]
+        return kk, vv, qs, kns, vns
+
+    step_s, sample, spent = oracle_sample_time(wl, get_unit, get_decode, st.budgets, st.n_keep,
+                                               target_s)
+    return {"value": round(wl.batch * wl.seq_len / step_s, 2), "unit": "tokens/s",
+            "cores": _threads(), "kind": "oracle", "sample": sample,
+            "sample_seconds": round(spent, 2), "step_seconds_extrapolated": round(step_s, 2)}
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the CPU oracle, timed on this host's cores, each step a
+    bounded sample of the workload extrapolated to a full step."""
+    if rank != 0:
+        return
+    import numpy as np
+    import torch
+
+    from oracle import ripple_oracle as O
+    from paper_2608_08684_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    G = wl.group
+    budgets = O.alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
+                              wl.global_budget)
+    n_keep = [O.keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    layer_cache = {}
+
+    def layer_tensors(layer):
+        if layer not in layer_cache:
+            layer_cache.clear()
+            layer_cache[layer] = (synth.layer_window_queries(wl, layer),
+                                  synth.layer_keys(wl, layer), synth.layer_values(wl, layer))
+        return layer_cache[layer]
+
+    def get_unit(layer, b, h):
+        q, k, v = layer_tensors(layer)
+        return (synth.to_f64(q[b, h * G:(h + 1) * G]), synth.to_f64(k[b, h]), synth.to_f64(v[b, h]))
+
+    def get_decode(layer, steps):
+        cap = n_keep[layer]
+        kc, vc = synth.decode_caches(wl.replace(batch=1, n_kv_heads=1), layer, cap)
+        dec = [synth.decode_inputs(wl.replace(batch=1), s, layers=[layer]) for s in range(steps)]
+        return (synth.to_f64(kc[0, 0]), synth.to_f64(vc[0, 0]),
+                [synth.to_f64(d[0][0, 0, 0:G]) for d in dec],
+                [synth.to_f64(d[1][0, 0, 0]) for d in dec], [synth.to_f64(d[2][0, 0, 0]) for d in dec])
+
+    per_step = max(2.0, min(args.cpu_seconds, 120.0 / max(1, args.steps + args.warmup)))
+    times, sample = [], ""
+    for i in range(args.warmup + args.steps):
+        step_s, sample, _ = oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, per_step)
+        if i >= args.warmup:
+            times.append(step_s)
+    step_s = statistics.mean(times)
+    value = wl.batch * wl.seq_len / step_s
+    line = {"metric": "compressed-prefill tokens/s; ragged decode-attn HBM GB/s vs GB300 peak",
+            "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name},
+            "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": _threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", str(args.gpus if args.gpus == 1 else 1)))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_ours(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,245 @@
+/*
+ * ripple.h -- C ABI of the RippleKV serving hot path on GB300 (sm_103a).
+ *
+ * RippleKV (arxiv 2608.08684) gives each layer l of a decoder a KV-cache
+ * budget b_l from a per-layer sensitivity profile, keeps only b_l cached
+ * positions of that layer (chosen by the base method's token scoring, SnapKV's
+ * observation window), and decodes against the compressed caches. This library
+ * implements that path: a host budget allocator (Sec. 4.4, Eqs. 9-12), a
+ * per-layer compression chain on the GPU (scoring, pooling, top-k selection,
+ * gather into a compact cache; Sec. 4.1 Eq. 4 and Sec. 4.4 last paragraph) and
+ * GQA decode attention over the ragged compressed caches (Sec. 4.1).
+ *
+ * Conventions for every entry point:
+ *   - Pointers named *_host are host memory; every other data pointer is CUDA
+ *     device memory owned by the caller. The library never allocates, frees or
+ *     keeps a reference to caller memory after a call returns.
+ *   - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *     stream. GPU work is enqueued on it in order; no call synchronises the
+ *     host with the device.
+ *   - Argument errors are detected on the host before anything is enqueued and
+ *     returned as a ripple_status; outputs are then untouched. Errors found by
+ *     the kernels (a full cache, a bounded wait that ran out, an index out of
+ *     range) are written to *dev_status (a device int32 the caller zeroes and
+ *     reads after synchronising the stream; the first error code written wins).
+ *     dev_status may be NULL, in which case device-side errors are not reported.
+ *   - dtype RIPPLE_BF16 means bfloat16 K/V/Q storage; RIPPLE_F32 means fp32.
+ *     Arithmetic is fp32 (tensor cores take bf16 operands with fp32
+ *     accumulation for the window-query/key contraction).
+ *   - All tensors are dense, row-major, with the innermost dimension the head
+ *     dimension d, and 16-byte aligned.
+ */
+#ifndef RIPPLE_H
+#define RIPPLE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RIPPLE_OK = 0,
+  RIPPLE_EINVAL = 1,     /* invalid argument (shape, value, alignment, NULL) */
+  RIPPLE_EWORKSPACE = 2, /* workspace smaller than the *_workspace_bytes query */
+  RIPPLE_EFULL = 3,      /* decode: a layer's cache had no free row to append */
+  RIPPLE_ECUDA = 4,      /* a CUDA runtime call failed (launch, attribute, ...) */
+  RIPPLE_ETIMEOUT = 5,   /* a bounded in-kernel wait ran out (device status) */
+  RIPPLE_EBOUNDS = 6     /* a kernel met an out-of-range index (device status) */
+} ripple_status;
+
+typedef enum { RIPPLE_F32 = 0, RIPPLE_BF16 = 1 } ripple_dtype;
+
+typedef enum {
+  RIPPLE_POOL_MAX = 0, /* max over the clipped window (default) */
+  RIPPLE_POOL_AVG = 1, /* mean over the clipped window, summed in index order */
+  RIPPLE_POOL_NONE = 2 /* votes used as they are */
+} ripple_pool;
+
+/* Largest number of layers one ripple_decode_attn call may cover. */
+#define RIPPLE_MAX_LAYERS 128
+
+/* ------------------------------------------------------------------------ */
+/* Budget allocation (host only).                                            */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * ripple_alloc_budgets -- per-layer cache budgets from a sensitivity profile.
+ *
+ * Sec. 4.4 and Algorithm 1 "Budget Allocation":
+ *   Eq. 9   s_hat_l = (s_l - s_min) / (s_max - s_min); all s_l equal -> s_hat = 0
+ *   Eq. 10  w~_l = exp(log(ratio) * s_hat_l)
+ *   Eq. 11  w = ClipNormalize(w~, gamma): clip to [1/gamma, gamma], then rescale
+ *           to mean one over the layers
+ *   Eq. 12  b_l = round(global_budget / n_layers * w_l), made to satisfy Eq. 5
+ *           (sum_l b_l = global_budget) by taking floor(quota_l) and giving one
+ *           more token to each of the global_budget - sum(floor) layers with
+ *           the largest fractional parts, ties to the lower layer index.
+ * The +epsilon of Algorithm 1's normalisation is not applied (Eq. 9 handles the
+ * identical case explicitly). Computed in IEEE double with libm exp/log, in
+ * layer order, without fused multiply-add: results are bit-reproducible.
+ *
+ * sens_host      [n_layers] sensitivity s_l (finite).
+ * n_layers       |A| >= 1.
+ * ratio          r >= 1, finite (r = 1 gives uniform budgets).
+ * gamma          clip bound >= 1; gamma <= 0 or +infinity disables clipping.
+ * global_budget  B >= 0, tokens summed over layers (per sequence and KV head).
+ * budgets_host   [n_layers] output b_l.
+ * Returns RIPPLE_EINVAL for NULL pointers, n_layers < 1, ratio < 1 or not
+ * finite, 0 < gamma < 1, NaN gamma, a non-finite s_l or global_budget < 0.
+ * Pure, reentrant, no CUDA calls.
+ */
+ripple_status ripple_alloc_budgets(const double *sens_host, int32_t n_layers, double ratio,
+                                   double gamma, int64_t global_budget,
+                                   int64_t *budgets_host);
+
+/*
+ * ripple_keep_count -- tokens one (batch, kv head) of a layer keeps:
+ * n = min(seq_len, max(budget, window)). The budget counts the observation
+ * window (SnapKV keeps the window; the paper's b_l = |S_l|, Eq. 4). Returns -1
+ * for seq_len < 1, window < 1, window > seq_len or budget < 0.
+ */
+int32_t ripple_keep_count(int64_t budget, int32_t seq_len, int32_t window);
+
+/* ------------------------------------------------------------------------ */
+/* Per-layer compression (prefill time).                                     */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  int32_t batch;       /* B >= 1 */
+  int32_t n_q_heads;   /* Hq, a multiple of n_kv_heads */
+  int32_t n_kv_heads;  /* Hkv >= 1; GQA group G = Hq / Hkv, G * window <= 256 */
+  int32_t head_dim;    /* d: 64 or 128 */
+  int32_t seq_len;     /* T >= 1, prompt tokens cached */
+  int32_t window;      /* w, 1 <= w <= min(T, 64): observation window (last w prompt queries) */
+  int32_t pool_kernel; /* odd, 1..31: 1-D pooling width over the prefix votes */
+  int32_t pool_type;   /* ripple_pool */
+  int32_t dtype;       /* ripple_dtype of q_win, k, v, k_out, v_out */
+  float scale;         /* logit scale; 0 means 1/sqrt(head_dim) */
+} ripple_layer_desc;
+
+/* Device workspace bytes ripple_compress_layer needs for this shape. */
+ripple_status ripple_compress_workspace_bytes(const ripple_layer_desc *desc, size_t *bytes_host);
+
+/*
+ * ripple_compress_layer -- compress one layer's KV cache to its budget.
+ *
+ * For every unit (b, h) (batch row, KV head), with P = T - w:
+ *  1. scores every cached token from the observation window (SnapKV rule kept
+ *     by RippleKV, Sec. 4.4 last paragraph): the G*w rows r = (query head
+ *     h*G + g, window position i) of q_win, at positions P + i, give logits
+ *     x[r][t] = scale * q_r . k_t for the keys t <= P + i they can see; each row
+ *     is softmax-normalised over its keys, and the vote of key t is the sum of
+ *     its probabilities over all G*w rows;
+ *  2. pools the prefix votes (t < P) with a stride-1 window of pool_kernel,
+ *     clipped to the prefix;
+ *  3. keeps the n - w prefix tokens with the largest pooled score (ties: lower
+ *     index), plus the w window tokens, n = ripple_keep_count(budget, T, w);
+ *  4. copies the kept K and V rows, in ascending token order, to rows 0..n-1 of
+ *     k_out / v_out (Eq. 4: compression only removes positions).
+ * If n == T every token is kept (no scoring needed) and k_out/v_out are copies.
+ *
+ * q_win      [B][Hq][w][d]   the last w prompt queries of this layer
+ * k, v       [B][Hkv][T][d]  this layer's prefill cache
+ * k_out,v_out[B][Hkv][cap][d] compressed caches; rows >= n are left untouched
+ * cap        rows per (b, h) of k_out/v_out, >= n (room for decode appends)
+ * idx_out    int32 [B][Hkv][n] kept token positions, ascending (device)
+ * scores_out fp32 [B][Hkv][P] unpooled votes of the prefix tokens, or NULL. When
+ *            n == T and scores_out is not NULL the votes are still computed.
+ * n_keep_host  receives n (host).
+ * workspace  device scratch of at least ripple_compress_workspace_bytes bytes,
+ *            256-byte aligned; its contents need no initialisation and are
+ *            meaningless after the call. Calls that share a workspace must be
+ *            ordered on the GPU (same stream, or events).
+ * Errors: RIPPLE_EINVAL (bad desc, budget < 0, cap < n, NULL or misaligned
+ * pointers), RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status: RIPPLE_ETIMEOUT.
+ */
+ripple_status ripple_compress_layer(const ripple_layer_desc *desc, int64_t budget,
+                                    const void *q_win, const void *k, const void *v,
+                                    void *k_out, void *v_out, int32_t cap,
+                                    int32_t *idx_out, float *scores_out,
+                                    int32_t *n_keep_host, void *workspace,
+                                    size_t workspace_bytes, int32_t *dev_status,
+                                    void *stream);
+
+/*
+ * ripple_select_layer -- steps 2-4 of ripple_compress_layer (pooling, top-k
+ * selection with the window appended, gather) from caller-provided votes
+ * instead of the window scoring. For scorers that produce the SnapKV votes
+ * elsewhere (for instance inside a fused prefill attention), and for checking
+ * the selection on chosen scores.
+ *
+ * votes      fp32 [B][Hkv][P] prefix votes (P = T - w), finite and >= 0.
+ * Other arguments as in ripple_compress_layer (q_win is not needed).
+ */
+ripple_status ripple_select_layer(const ripple_layer_desc *desc, int64_t budget,
+                                  const float *votes, const void *k, const void *v,
+                                  void *k_out, void *v_out, int32_t cap, int32_t *idx_out,
+                                  int32_t *n_keep_host, void *workspace, size_t workspace_bytes,
+                                  int32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Decoding against the ragged compressed caches.                            */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  int32_t n_layers;   /* layers covered by this call, 1..RIPPLE_MAX_LAYERS */
+  int32_t batch;      /* B */
+  int32_t n_q_heads;  /* Hq, a multiple of n_kv_heads, G = Hq/Hkv <= 8 */
+  int32_t n_kv_heads; /* Hkv */
+  int32_t head_dim;   /* d: 64 or 128 */
+  int32_t dtype;      /* ripple_dtype of q, k_new, v_new and the caches */
+  float scale;        /* logit scale; 0 means 1/sqrt(head_dim) */
+} ripple_decode_desc;
+
+/* Device workspace bytes ripple_decode_attn needs for these layers' capacities. */
+ripple_status ripple_decode_workspace_bytes(const ripple_decode_desc *desc,
+                                            const int32_t *caps_host, size_t *bytes_host);
+
+/*
+ * ripple_decode_attn -- one decode step over several layers in one launch.
+ *
+ * Sec. 4.1: during decoding each new query attends to the cached states. For
+ * every layer l, batch row b and KV head h, with len = lens[l]:
+ *   1. appends the new key/value rows k_new[l][b][h], v_new[l][b][h] at row len
+ *      of that layer's caches;
+ *   2. for each of the G query heads of the group, attends over rows 0..len
+ *      (the retained tokens, earlier appended tokens and the new token):
+ *      out = sum_j softmax_j(scale * q . k_j) v_j, fp32 accumulation;
+ *   3. after all layers are done, lens[l] = len + 1.
+ * The query positions are not rotated (keys are stored post-rotation).
+ *
+ * q            [L][B][Hq][d]
+ * k_new, v_new [L][B][Hkv][d]
+ * k_caches_host, v_caches_host  host arrays of L device pointers; layer l's
+ *              caches are [B][Hkv][caps_host[l]][d]
+ * caps_host    host [L], rows per (b, h) of each layer's caches
+ * lens         device int32 [L]: rows in use per layer (same for every b, h);
+ *              read, then incremented by one per layer
+ * out          device fp32 [L][B][Hq][d]
+ * workspace    device scratch of at least ripple_decode_workspace_bytes bytes
+ * A layer with lens[l] >= caps_host[l] (or lens[l] < 0) is not appended to,
+ * its output rows are zero, its length is unchanged, and RIPPLE_EFULL is
+ * written to *dev_status.
+ * Errors: RIPPLE_EINVAL, RIPPLE_EWORKSPACE, RIPPLE_ECUDA.
+ */
+ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
+                                 const void *k_new, const void *v_new,
+                                 void *const *k_caches_host, void *const *v_caches_host,
+                                 const int32_t *caps_host, int32_t *lens, float *out,
+                                 void *workspace, size_t workspace_bytes,
+                                 int32_t *dev_status, void *stream);
+
+/* Number of kernels this library has launched in this process so far
+ * (host-side count of launch calls; for benchmarks and launch accounting). */
+uint64_t ripple_kernel_launches(void);
+
+/* Human-readable name of a status code (static string). */
+const char *ripple_status_string(int32_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RIPPLE_H */

@@ -1,0 +1,156 @@
+// ripple_compress_layer: the per-layer compression chain (Sec. 4.1 Eq. 4 and
+// Sec. 4.4 last paragraph: RippleKV keeps the base method's scoring and
+// selection and changes only the number of tokens each layer keeps).
+//   scoring   -> votes [units][P]     (tcgen05 for bf16 d=128, fp32 SIMT otherwise)
+//   selection -> idx   [units][n]     (pooling + exact top-k, window appended)
+//   gather    -> k_out, v_out [units][cap][d]
+// Everything is enqueued on the caller's stream; nothing synchronises.
+#include <math.h>
+
+#include <atomic>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace ripple {
+
+static size_t round_up(size_t x) { return (x + 255) & ~(size_t)255; }
+
+static std::atomic<uint64_t> g_launches{0};
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+CompressWs carve_compress_ws(const LayerGeom &g, void *base) {
+  CompressWs w{};
+  uint8_t *p = (uint8_t *)base;
+  size_t off = 0;
+  const size_t n_chunks = (g.T + kScoreChunk - 1) / kScoreChunk;
+  auto take = [&](size_t bytes) {
+    uint8_t *r = p ? p + off : nullptr;
+    off += round_up(bytes);
+    return r;
+  };
+  w.row_partial = (float2 *)take(sizeof(float2) * g.units * n_chunks * g.R);
+  w.row_lognorm = (float *)take(sizeof(float) * g.units * g.R);
+  w.votes = (float *)take(sizeof(float) * g.units * (size_t)g.P);
+  w.keys = (uint32_t *)take(g.P > kSelectSmemKeys ? sizeof(uint32_t) * g.units * (size_t)g.P : 0);
+  w.counters = (int32_t *)take(1024);
+  w.bytes = off;
+  return w;
+}
+
+static bool make_geom(const ripple_layer_desc *d, LayerGeom *g) {
+  if (d == nullptr) return false;
+  if (d->batch < 1 || d->n_q_heads < 1 || d->n_kv_heads < 1) return false;
+  if (d->n_q_heads % d->n_kv_heads != 0) return false;
+  if (d->head_dim != 64 && d->head_dim != 128) return false;
+  if (d->seq_len < 1 || d->window < 1 || d->window > d->seq_len || d->window > 64) return false;
+  if (d->pool_kernel < 1 || d->pool_kernel > 31 || (d->pool_kernel & 1) == 0) return false;
+  if (d->pool_type != RIPPLE_POOL_MAX && d->pool_type != RIPPLE_POOL_AVG &&
+      d->pool_type != RIPPLE_POOL_NONE)
+    return false;
+  if (d->dtype != RIPPLE_F32 && d->dtype != RIPPLE_BF16) return false;
+  if (!(d->scale >= 0.f) || isinf(d->scale)) return false;
+  const int G = d->n_q_heads / d->n_kv_heads;
+  if (G * d->window > 256) return false;
+  if ((int64_t)d->batch * d->n_kv_heads > 65535) return false;
+  g->B = d->batch;
+  g->Hq = d->n_q_heads;
+  g->Hkv = d->n_kv_heads;
+  g->G = G;
+  g->D = d->head_dim;
+  g->T = d->seq_len;
+  g->W = d->window;
+  g->P = d->seq_len - d->window;
+  g->R = G * d->window;
+  g->units = d->batch * d->n_kv_heads;
+  g->dtype = d->dtype;
+  g->pool_kernel = d->pool_kernel;
+  g->pool_type = d->pool_type;
+  const float scale = d->scale > 0.f ? d->scale : 1.0f / sqrtf((float)d->head_dim);
+  g->scale2 = scale * kLog2e;
+  return true;
+}
+
+}  // namespace ripple
+
+using namespace ripple;
+
+extern "C" uint64_t ripple_kernel_launches(void) { return g_launches.load(); }
+
+extern "C" ripple_status ripple_compress_workspace_bytes(const ripple_layer_desc *desc,
+                                                         size_t *bytes_host) {
+  LayerGeom g;
+  if (!make_geom(desc, &g) || bytes_host == nullptr) return RIPPLE_EINVAL;
+  *bytes_host = carve_compress_ws(g, nullptr).bytes;
+  return RIPPLE_OK;
+}
+
+extern "C" ripple_status ripple_compress_layer(const ripple_layer_desc *desc, int64_t budget,
+                                               const void *q_win, const void *k, const void *v,
+                                               void *k_out, void *v_out, int32_t cap,
+                                               int32_t *idx_out, float *scores_out,
+                                               int32_t *n_keep_host, void *workspace,
+                                               size_t workspace_bytes, int32_t *dev_status,
+                                               void *stream) {
+  LayerGeom g;
+  if (!make_geom(desc, &g)) return RIPPLE_EINVAL;
+  if (budget < 0 || !q_win || !k || !v || !k_out || !v_out || !idx_out || !n_keep_host ||
+      !workspace)
+    return RIPPLE_EINVAL;
+  auto aligned = [](const void *p) { return ((uintptr_t)p & 15u) == 0; };
+  if (!aligned(q_win) || !aligned(k) || !aligned(v) || !aligned(k_out) || !aligned(v_out) ||
+      !aligned(idx_out) || (scores_out && !aligned(scores_out)) || ((uintptr_t)workspace & 255u))
+    return RIPPLE_EINVAL;
+  const int n = ripple_keep_count(budget, g.T, g.W);
+  if (n < 0 || cap < n) return RIPPLE_EINVAL;
+  const CompressWs ws = carve_compress_ws(g, workspace);
+  if (workspace_bytes < ws.bytes) return RIPPLE_EWORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+
+  const bool keep_all = (n == g.T);
+  float *votes = scores_out ? scores_out : ws.votes;
+  if (g.P > 0 && (!keep_all || scores_out)) {
+    cudaError_t e = score_tc_supported(g)
+                        ? launch_score_tc(g, q_win, k, ws, votes, dev_status, st)
+                        : launch_score_simt(g, q_win, k, ws, votes, st);
+    RIPPLE_CUDA_TRY(e);
+  }
+  if (keep_all) {
+    RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
+  } else {
+    RIPPLE_CUDA_TRY(launch_select(g, votes, ws, n, idx_out, st));
+  }
+  RIPPLE_CUDA_TRY(launch_gather(g, k, v, idx_out, n, k_out, v_out, cap, dev_status, st));
+  *n_keep_host = n;
+  return RIPPLE_OK;
+}
+
+extern "C" ripple_status ripple_select_layer(const ripple_layer_desc *desc, int64_t budget,
+                                             const float *votes, const void *k, const void *v,
+                                             void *k_out, void *v_out, int32_t cap,
+                                             int32_t *idx_out, int32_t *n_keep_host,
+                                             void *workspace, size_t workspace_bytes,
+                                             int32_t *dev_status, void *stream) {
+  LayerGeom g;
+  if (!make_geom(desc, &g)) return RIPPLE_EINVAL;
+  if (budget < 0 || !votes || !k || !v || !k_out || !v_out || !idx_out || !n_keep_host ||
+      !workspace)
+    return RIPPLE_EINVAL;
+  auto aligned = [](const void *p) { return ((uintptr_t)p & 15u) == 0; };
+  if (!aligned(votes) || !aligned(k) || !aligned(v) || !aligned(k_out) || !aligned(v_out) ||
+      !aligned(idx_out) || ((uintptr_t)workspace & 255u))
+    return RIPPLE_EINVAL;
+  const int n = ripple_keep_count(budget, g.T, g.W);
+  if (n < 0 || cap < n) return RIPPLE_EINVAL;
+  const CompressWs ws = carve_compress_ws(g, workspace);
+  if (workspace_bytes < ws.bytes) return RIPPLE_EWORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (n == g.T) {
+    RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
+  } else {
+    RIPPLE_CUDA_TRY(launch_select(g, votes, ws, n, idx_out, st));
+  }
+  RIPPLE_CUDA_TRY(launch_gather(g, k, v, idx_out, n, k_out, v_out, cap, dev_status, st));
+  *n_keep_host = n;
+  return RIPPLE_OK;
+}

@@ -1,0 +1,57 @@
+// Host-side launchers shared between the translation units of libripple.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "ripple.h"
+
+namespace ripple {
+
+// Host-side count of kernel launches (ripple_kernel_launches).
+void count_launches(int n);
+
+// Geometry of one layer's compression, derived from ripple_layer_desc.
+struct LayerGeom {
+  int B, Hq, Hkv, G, D, T, W, P, R;  // R = G * W window rows per unit
+  int units;                          // B * Hkv
+  int dtype;
+  int pool_kernel, pool_type;
+  float scale2;                       // logit scale * log2(e)
+};
+
+constexpr int kScoreChunk = 128;      // keys per scoring work item
+constexpr int kSelectThreads = 1024;  // threads of the selection CTA
+constexpr int kSelectSmemKeys = 48 * 1024;  // prefix lengths up to this keep keys in smem
+
+// Workspace carve-up of one compression call.
+struct CompressWs {
+  float2 *row_partial;  // [units][n_chunks][R] (max, sum) in the log2 domain
+  float *row_lognorm;   // [units][R] max + log2(sum), log2 domain
+  float *votes;         // [units][P] unpooled votes (when scores_out is NULL)
+  uint32_t *keys;       // [units][P] pooled-score sort keys (long prefixes only)
+  int32_t *counters;    // small control block
+  size_t bytes;
+};
+CompressWs carve_compress_ws(const LayerGeom &g, void *base);
+
+// Scoring, SIMT fp32 path (any dtype).
+cudaError_t launch_score_simt(const LayerGeom &g, const void *q_win, const void *k,
+                              const CompressWs &ws, float *votes, cudaStream_t st);
+// Scoring, tcgen05 tensor-core path (bf16, d = 128).
+bool score_tc_supported(const LayerGeom &g);
+cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
+                            const CompressWs &ws, float *votes, int32_t *status,
+                            cudaStream_t st);
+// Pooling + exact top-k per unit; writes idx [units][n].
+cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
+                          int n_keep, int32_t *idx, cudaStream_t st);
+// idx = 0..T-1 for every unit (keep-all case).
+cudaError_t launch_iota(const LayerGeom &g, int32_t *idx, cudaStream_t st);
+// Gather kept K and V rows into [units][cap][d].
+cudaError_t launch_gather(const LayerGeom &g, const void *k, const void *v, const int32_t *idx,
+                          int n_keep, void *k_out, void *v_out, int cap, int32_t *status,
+                          cudaStream_t st);
+
+}  // namespace ripple

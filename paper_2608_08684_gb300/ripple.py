@@ -1,0 +1,208 @@
+"""Python binding of libripple.so (the C ABI declared in include/ripple.h).
+
+Argument marshalling only: every function here passes raw pointers, sizes and
+the current CUDA stream to the entry point of the same name, and raises
+RippleError on a non-zero status. All computation happens in the library's
+kernels (or, for ripple_alloc_budgets, in its host C code). Importing this
+module fails loudly if the library has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import torch
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libripple.so")
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is not built: call paper_2608_08684_gb300.build.build_library()")
+_lib = ctypes.CDLL(LIB_PATH)
+
+F32, BF16 = 0, 1
+POOL_MAX, POOL_AVG, POOL_NONE = 0, 1, 2
+OK, EINVAL, EWORKSPACE, EFULL, ECUDA, ETIMEOUT, EBOUNDS = range(7)
+MAX_LAYERS = 128
+_POOLS = {"max": POOL_MAX, "avg": POOL_AVG, "none": POOL_NONE}
+_DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
+
+
+class RippleError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+class LayerDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("seq_len", ctypes.c_int32), ("window", ctypes.c_int32),
+                ("pool_kernel", ctypes.c_int32), ("pool_type", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
+class DecodeDesc(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("batch", ctypes.c_int32),
+                ("n_q_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("scale", ctypes.c_float)]
+
+
+_p = ctypes.c_void_p
+_i32, _i64, _f64, _sz = ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_size_t
+
+_lib.ripple_alloc_budgets.argtypes = [ctypes.POINTER(_f64), _i32, _f64, _f64, _i64,
+                                      ctypes.POINTER(_i64)]
+_lib.ripple_alloc_budgets.restype = _i32
+_lib.ripple_keep_count.argtypes = [_i64, _i32, _i32]
+_lib.ripple_keep_count.restype = _i32
+_lib.ripple_compress_workspace_bytes.argtypes = [ctypes.POINTER(LayerDesc), ctypes.POINTER(_sz)]
+_lib.ripple_compress_workspace_bytes.restype = _i32
+_lib.ripple_compress_layer.argtypes = [ctypes.POINTER(LayerDesc), _i64, _p, _p, _p, _p, _p, _i32,
+                                       _p, _p, ctypes.POINTER(_i32), _p, _sz, _p, _p]
+_lib.ripple_compress_layer.restype = _i32
+_lib.ripple_select_layer.argtypes = [ctypes.POINTER(LayerDesc), _i64, _p, _p, _p, _p, _p, _i32, _p,
+                                     ctypes.POINTER(_i32), _p, _sz, _p, _p]
+_lib.ripple_select_layer.restype = _i32
+_lib.ripple_decode_workspace_bytes.argtypes = [ctypes.POINTER(DecodeDesc), ctypes.POINTER(_i32),
+                                               ctypes.POINTER(_sz)]
+_lib.ripple_decode_workspace_bytes.restype = _i32
+_lib.ripple_decode_attn.argtypes = [ctypes.POINTER(DecodeDesc), _p, _p, _p, ctypes.POINTER(_p),
+                                    ctypes.POINTER(_p), ctypes.POINTER(_i32), _p, _p, _p, _sz, _p,
+                                    _p]
+_lib.ripple_decode_attn.restype = _i32
+_lib.ripple_kernel_launches.argtypes = []
+_lib.ripple_kernel_launches.restype = ctypes.c_uint64
+_lib.ripple_status_string.argtypes = [_i32]
+_lib.ripple_status_string.restype = ctypes.c_char_p
+
+
+def status_string(status: int) -> str:
+    return _lib.ripple_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise RippleError(status, where)
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+def layer_desc(batch, n_q_heads, n_kv_heads, head_dim, seq_len, window, pool_kernel=7,
+               pool="max", dtype=torch.bfloat16, scale=0.0) -> LayerDesc:
+    return LayerDesc(batch, n_q_heads, n_kv_heads, head_dim, seq_len, window, pool_kernel,
+                     _POOLS[pool], _DTYPES[dtype], scale)
+
+
+def decode_desc(n_layers, batch, n_q_heads, n_kv_heads, head_dim, dtype=torch.bfloat16,
+                scale=0.0) -> DecodeDesc:
+    return DecodeDesc(n_layers, batch, n_q_heads, n_kv_heads, head_dim, _DTYPES[dtype], scale)
+
+
+# ----------------------------------------------------------------- entry points
+
+
+def ripple_alloc_budgets(sens, ratio: float, gamma: float, global_budget: int) -> list:
+    """Per-layer budgets b_l (Eqs. 9-12 with Eq. 5), computed by the host C allocator."""
+    n = len(sens)
+    s = (_f64 * n)(*[float(x) for x in sens])
+    out = (_i64 * n)()
+    _check(_lib.ripple_alloc_budgets(s, n, float(ratio), float(gamma), int(global_budget), out),
+           "ripple_alloc_budgets")
+    return [int(x) for x in out]
+
+
+def ripple_keep_count(budget: int, seq_len: int, window: int) -> int:
+    n = _lib.ripple_keep_count(int(budget), int(seq_len), int(window))
+    if n < 0:
+        raise RippleError(EINVAL, "ripple_keep_count")
+    return n
+
+
+def ripple_compress_workspace_bytes(desc: LayerDesc) -> int:
+    out = _sz()
+    _check(_lib.ripple_compress_workspace_bytes(ctypes.byref(desc), ctypes.byref(out)),
+           "ripple_compress_workspace_bytes")
+    return out.value
+
+
+def ripple_compress_layer(desc: LayerDesc, budget: int, q_win, k, v, k_out, v_out, idx_out,
+                          workspace, scores_out=None, dev_status=None, stream=None) -> int:
+    """Compress one layer; returns n, the tokens kept per (batch, kv head).
+
+    k_out/v_out are [B][Hkv][cap][d]; idx_out holds at least B*Hkv*n int32.
+    """
+    cap = k_out.shape[-2]
+    n = _i32()
+    _check(_lib.ripple_compress_layer(ctypes.byref(desc), int(budget), _ptr(q_win), _ptr(k),
+                                      _ptr(v), _ptr(k_out), _ptr(v_out), cap, _ptr(idx_out),
+                                      _ptr(scores_out), ctypes.byref(n), _ptr(workspace),
+                                      workspace.numel() * workspace.element_size(),
+                                      _ptr(dev_status), _stream(stream)),
+           "ripple_compress_layer")
+    return n.value
+
+
+def ripple_select_layer(desc: LayerDesc, budget: int, votes, k, v, k_out, v_out, idx_out,
+                        workspace, dev_status=None, stream=None) -> int:
+    """Pool, select and gather one layer from given fp32 votes [B][Hkv][P]; returns n."""
+    cap = k_out.shape[-2]
+    n = _i32()
+    _check(_lib.ripple_select_layer(ctypes.byref(desc), int(budget), _ptr(votes), _ptr(k), _ptr(v),
+                                    _ptr(k_out), _ptr(v_out), cap, _ptr(idx_out), ctypes.byref(n),
+                                    _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                    _ptr(dev_status), _stream(stream)),
+           "ripple_select_layer")
+    return n.value
+
+
+def ripple_decode_workspace_bytes(desc: DecodeDesc, caps) -> int:
+    c = (_i32 * len(caps))(*[int(x) for x in caps])
+    out = _sz()
+    _check(_lib.ripple_decode_workspace_bytes(ctypes.byref(desc), c, ctypes.byref(out)),
+           "ripple_decode_workspace_bytes")
+    return out.value
+
+
+class DecodeTables:
+    """Host arrays (cache pointers, capacities) of ripple_decode_attn, built once."""
+
+    def __init__(self, k_caches, v_caches):
+        L = len(k_caches)
+        self.k = (_p * L)(*[_ptr(t) for t in k_caches])
+        self.v = (_p * L)(*[_ptr(t) for t in v_caches])
+        self.caps = (_i32 * L)(*[int(t.shape[-2]) for t in k_caches])
+        self._keep = (list(k_caches), list(v_caches))
+
+
+def ripple_decode_attn(desc: DecodeDesc, q, k_new, v_new, tables: DecodeTables, lens, out,
+                       workspace, dev_status=None, stream=None):
+    """One decode step over desc.n_layers layers: append, attend, advance lens."""
+    _check(_lib.ripple_decode_attn(ctypes.byref(desc), _ptr(q), _ptr(k_new), _ptr(v_new),
+                                   tables.k, tables.v, tables.caps, _ptr(lens), _ptr(out),
+                                   _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                   _ptr(dev_status), _stream(stream)),
+           "ripple_decode_attn")
+
+
+def ripple_kernel_launches() -> int:
+    """Kernels the library has launched in this process."""
+    return int(_lib.ripple_kernel_launches())
+
+
+def default_scale(head_dim: int) -> float:
+    return 1.0 / math.sqrt(head_dim)

@@ -39,7 +39,8 @@ def _splitmix64(x: int) -> int:
     return x ^ (x >> 31)
 
 
-_TAGS = {"k": 1, "v": 2, "q_win": 3, "scale": 4, "dq": 5, "dk": 6, "dv": 7, "sens": 8}
+_TAGS = {"k": 1, "v": 2, "q_win": 3, "scale": 4, "dq": 5, "dk": 6, "dv": 7, "sens": 8,
+         "votes": 9, "ck": 10, "cv": 11}
 
 
 def stream_seed(seed: int, tag: str, layer: int = 0, step: int = 0) -> int:
@@ -211,3 +212,27 @@ def decode_inputs(wl: Workload, step: int, device="cpu", layers=None):
 def to_f64(t: torch.Tensor) -> np.ndarray:
     """Exact float64 copy of a tensor's values (bf16 and fp32 embed exactly)."""
     return t.detach().to("cpu", torch.float64).numpy()
+
+
+def synthetic_votes(seed: int, units: int, prefix: int, levels: int = 0, device="cpu") -> torch.Tensor:
+    """fp32 [units][prefix] non-negative vote arrays for selection checks.
+
+    levels > 0 quantises the values to that many levels, which makes many exact
+    ties; levels == 0 keeps continuous values.
+    """
+    g = _generator(device, seed, "votes")
+    x = torch.rand((units, prefix), generator=g, device=device, dtype=torch.float32)
+    if levels > 0:
+        x = torch.floor(x * levels) / levels
+    return x * 0.01
+
+
+def decode_caches(wl: Workload, layer: int, cap: int, device="cpu"):
+    """Seeded K/V caches [B][Hkv][cap][d] of one layer for decode checks
+    (keys with the layer's channel scales, values N(0, 1))."""
+    shape = (wl.batch, wl.n_kv_heads, cap, wl.head_dim)
+    k = _normal(shape, _generator(device, wl.seed, "ck", layer), device)
+    if wl.kv_dist == "scaled_sinks":
+        k.mul_(channel_scales(wl, layer, device)[None, :, None, :])
+    v = _normal(shape, _generator(device, wl.seed, "cv", layer), device)
+    return k.to(wl.torch_dtype), v.to(wl.torch_dtype)

@@ -1,0 +1,116 @@
+"""The C-ABI library without a GPU: it loads, exports every declared symbol,
+its host allocator matches the oracle bit for bit, and host-side argument
+validation rejects bad calls before any CUDA work."""
+import ctypes
+import math
+import os
+import random
+import re
+
+import pytest
+
+from oracle import ripple_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names += re.findall(r"^\s*[A-Za-z_][\w\s\*]*?\b(ripple_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = _declared_functions()
+    for n in ("ripple_alloc_budgets", "ripple_compress_layer", "ripple_decode_attn"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(lib.LIB_PATH)
+    for name in _declared_functions():
+        assert hasattr(raw, name), name
+
+
+def _cases():
+    rnd = random.Random(2024)
+    out = []
+    for _ in range(300):
+        L = rnd.choice([1, 2, 3, 4, 5, 8, 31, 32, 80, 128])
+        kind = rnd.random()
+        if kind < 0.1:
+            s = [0.25] * L
+        elif kind < 0.2:
+            s = [float(rnd.randint(0, 3)) for _ in range(L)]
+        else:
+            s = [rnd.lognormvariate(-4.0, 1.2) for _ in range(L)]
+        r = rnd.choice([1.0, 1.25, 1.5, 1.75, 2.0, 4.0, 8.0, 32.0])
+        gamma = rnd.choice([math.inf, 0.0, -1.0, 1.0, 1.5, 2.0, 4.0])
+        B = rnd.choice([0, 1, 7, L, 3 * L + 1, 128 * L, 512 * L, 1024 * L + 13, 2048 * L])
+        out.append((s, r, gamma, B))
+    return out
+
+
+def test_host_allocator_bit_exact_vs_oracle(lib):
+    for s, r, gamma, B in _cases():
+        assert lib.ripple_alloc_budgets(s, r, gamma, B) == O.alloc_budgets(s, r, gamma, B)
+
+
+def test_host_allocator_worked_example(lib):
+    assert lib.ripple_alloc_budgets([0.2, 1.0, 0.6, 0.1], 4.0, math.inf, 512) == [72, 246, 133, 61]
+
+
+@pytest.mark.parametrize("args", [
+    ([], 4.0, math.inf, 10),
+    ([0.1, 0.2], 0.5, math.inf, 10),
+    ([0.1, 0.2], math.inf, math.inf, 10),
+    ([0.1, 0.2], math.nan, math.inf, 10),
+    ([0.1, 0.2], 4.0, 0.5, 10),
+    ([0.1, 0.2], 4.0, math.nan, 10),
+    ([0.1, math.nan], 4.0, math.inf, 10),
+    ([0.1, math.inf], 4.0, math.inf, 10),
+    ([0.1, 0.2], 4.0, math.inf, -1),
+])
+def test_host_allocator_rejects_bad_arguments(lib, args):
+    with pytest.raises(lib.RippleError) as e:
+        lib.ripple_alloc_budgets(*args)
+    assert e.value.status == lib.EINVAL
+
+
+def test_keep_count_matches_oracle(lib):
+    for b, T, w in [(100, 512, 32), (10, 512, 32), (5000, 512, 32), (0, 16, 16), (33, 33, 1)]:
+        assert lib.ripple_keep_count(b, T, w) == O.keep_count(b, T, w)
+    with pytest.raises(lib.RippleError):
+        lib.ripple_keep_count(5, 10, 11)
+
+
+def test_workspace_query_and_validation(lib):
+    d = lib.layer_desc(4, 32, 8, 128, 32768, 32)
+    assert lib.ripple_compress_workspace_bytes(d) > 4 * 8 * 32736 * 4
+    bad = [lib.layer_desc(1, 6, 4, 128, 100, 8),   # Hq not a multiple of Hkv
+           lib.layer_desc(1, 4, 2, 96, 100, 8),    # unsupported head_dim
+           lib.layer_desc(1, 4, 2, 64, 100, 101),  # window > T
+           lib.layer_desc(1, 4, 2, 64, 100, 8, pool_kernel=4),
+           lib.layer_desc(1, 64, 1, 64, 100, 8)]   # G * w > 256
+    for d in bad:
+        with pytest.raises(lib.RippleError):
+            lib.ripple_compress_workspace_bytes(d)
+
+
+def test_entry_points_reject_before_any_cuda_work(lib):
+    # NULL pointers / bad shapes are refused on the host; nothing is launched.
+    raw = lib._lib
+    d = lib.layer_desc(1, 4, 2, 64, 512, 32, dtype=__import__("torch").float32)
+    n = ctypes.c_int32(-7)
+    st = raw.ripple_compress_layer(ctypes.byref(d), 100, None, None, None, None, None, 128, None,
+                                   None, ctypes.byref(n), None, 0, None, None)
+    assert st == lib.EINVAL and n.value == -7
+    dd = lib.decode_desc(2, 1, 4, 2, 64)
+    st = raw.ripple_decode_attn(ctypes.byref(dd), None, None, None, None, None, None, None, None,
+                                None, 0, None, None)
+    assert st == lib.EINVAL
+    assert lib.status_string(lib.EFULL) == "cache full"

@@ -1,0 +1,154 @@
+"""GPU parity of the compression path (ripple_compress_layer, ripple_select_layer)
+against the CPU oracle on seeded inputs: votes within 1e-3 relative, retained
+sets agreeing on >= 99.9% of tokens with every difference inside the score
+tolerance, gathered rows byte-exact, selection bit-exact on shared votes."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import ripple_oracle as O
+from paper_2608_08684_gb300 import synth
+from tests import gpu_common as C
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def _check_layer(lib, wl, layer, budget, units="all", pool="max", scale=0.0, on_device=False):
+    gen = DEV if on_device else "cpu"
+    q_win, k, v = C.layer_inputs(wl, layer, gen)
+    dq, dk, dv = (t.to(DEV) for t in (q_win, k, v))
+    out = C.run_compress(lib, wl, budget, dq, dk, dv, cap_extra=3, pool=pool, scale=scale)
+    assert int(out["status"].item()) == 0
+    pairs = ([(b, h) for b in range(wl.batch) for h in range(wl.n_kv_heads)]
+             if units == "all" else units)
+    agree = total = 0
+    for b, h in pairs:
+        a, t = C.check_compress_unit(wl, out, dq, dk, dv, b, h, budget, pool,
+                                     scale if scale > 0 else None)
+        agree += a
+        total += t
+    return agree, total, out
+
+
+def test_tiny_workload_all_layers(lib):
+    wl = synth.WORKLOADS["tiny"]
+    s = synth.sensitivity_profile(wl)
+    budgets = lib.ripple_alloc_budgets(s, wl.ratio, wl.gamma, wl.global_budget)
+    assert budgets == O.alloc_budgets(s, wl.ratio, wl.gamma, wl.global_budget)
+    assert budgets == [72, 246, 133, 61]
+    agree = total = 0
+    for layer in range(wl.n_layers):
+        a, t, _ = _check_layer(lib, wl, layer, budgets[layer])
+        agree += a
+        total += t
+    assert agree >= 0.999 * total
+
+
+SMALL = [
+    # name, overrides
+    ("bf16-d128-G4-ragged", dict(batch=2, n_q_heads=8, n_kv_heads=2, head_dim=128, seq_len=1000,
+                                 dtype="bf16", kv_dist="scaled_sinks", seed=11), 200),
+    ("bf16-d128-G8", dict(batch=1, n_q_heads=16, n_kv_heads=2, head_dim=128, seq_len=700,
+                          dtype="bf16", kv_dist="scaled_sinks", seed=12), 300),
+    ("bf16-d64-G3-w7", dict(batch=1, n_q_heads=6, n_kv_heads=2, head_dim=64, seq_len=389,
+                            window=7, dtype="bf16", seed=13), 100),
+    ("f32-d128-G2", dict(batch=2, n_q_heads=4, n_kv_heads=2, head_dim=128, seq_len=300,
+                         dtype="f32", seed=14), 64),
+    ("bf16-one-tile-plus", dict(batch=1, n_q_heads=4, n_kv_heads=1, head_dim=128, seq_len=130,
+                                dtype="bf16", seed=15), 40),
+    ("bf16-G1-w1", dict(batch=3, n_q_heads=2, n_kv_heads=2, head_dim=128, seq_len=257, window=1,
+                        dtype="bf16", seed=16), 17),
+]
+
+
+@pytest.mark.parametrize("name,over,budget", SMALL, ids=[c[0] for c in SMALL])
+def test_small_shapes(lib, name, over, budget):
+    wl = synth.WORKLOADS["tiny"].replace(**over)
+    agree, total, _ = _check_layer(lib, wl, 0, budget)
+    assert agree >= 0.999 * total
+
+
+@pytest.mark.parametrize("budget", [0, 5, 32, 33, 479, 480, 511, 512, 513, 10**9])
+def test_budget_edges(lib, budget):
+    # budget below the window keeps the window only; budget >= T keeps all (Eq. 4)
+    wl = synth.WORKLOADS["tiny"]
+    agree, total, out = _check_layer(lib, wl, 1, budget)
+    assert out["n"] == O.keep_count(budget, wl.seq_len, wl.window)
+    assert agree >= 0.999 * total
+
+
+def test_keep_all_copies_cache_exactly(lib):
+    wl = synth.WORKLOADS["tiny"].replace(dtype="bf16", head_dim=128, seed=21)
+    q_win, k, v = (t.to(DEV) for t in C.layer_inputs(wl, 0, "cpu"))
+    out = C.run_compress(lib, wl, wl.seq_len + 7, q_win, k, v)
+    assert torch.equal(out["k_out"], k) and torch.equal(out["v_out"], v)
+
+
+@pytest.mark.parametrize("pool", ["avg", "none"])
+def test_pool_variants(lib, pool):
+    wl = synth.WORKLOADS["tiny"]
+    agree, total, _ = _check_layer(lib, wl, 2, 150, pool=pool)
+    assert agree >= 0.999 * total
+
+
+def test_custom_scale(lib):
+    wl = synth.WORKLOADS["tiny"]
+    agree, total, _ = _check_layer(lib, wl, 0, 100, scale=0.3)
+    assert agree >= 0.999 * total
+
+
+@pytest.mark.parametrize("T,w", [(1, 1), (32, 32), (40, 32)])
+def test_tiny_sequences(lib, T, w):
+    wl = synth.WORKLOADS["tiny"].replace(seq_len=T, window=w)
+    agree, total, _ = _check_layer(lib, wl, 0, 1)
+    assert agree >= 0.999 * total
+
+
+@pytest.mark.parametrize("units,P,levels,budget", [
+    (3, 480, 7, 100), (2, 4000, 50, 1000), (4, 100, 0, 60), (1, 60000, 300, 9000),
+    (2, 1025, 1, 500), (1, 5, 2, 10),
+])
+def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget):
+    # identical votes on both sides: selection and gather must agree bit for bit
+    w = 8
+    wl = synth.WORKLOADS["tiny"].replace(batch=1, n_q_heads=units, n_kv_heads=units,
+                                         head_dim=64, seq_len=P + w, window=w, dtype="bf16")
+    votes = synth.synthetic_votes(31 + P, units, P, levels)
+    k = synth.layer_keys(wl, 0)
+    v = synth.layer_values(wl, 0)
+    desc = lib.layer_desc(1, units, units, 64, P + w, w, 7, "max", torch.bfloat16)
+    n = lib.ripple_keep_count(budget, P + w, w)
+    k_out = torch.zeros(1, units, n, 64, dtype=torch.bfloat16, device=DEV)
+    v_out = torch.zeros_like(k_out)
+    idx = torch.empty(units * n, dtype=torch.int32, device=DEV)
+    ws = torch.empty(lib.ripple_compress_workspace_bytes(desc), dtype=torch.uint8, device=DEV)
+    assert lib.ripple_select_layer(desc, budget, votes.to(DEV), k.to(DEV), v.to(DEV), k_out,
+                                   v_out, idx, ws) == n
+    torch.cuda.synchronize()
+    idx = idx.view(units, n).cpu().numpy()
+    for u in range(units):
+        pooled = O.pool_scores(votes[u].numpy(), 7, "max")
+        expect = O.select_tokens(pooled, n, P + w, w)
+        np.testing.assert_array_equal(idx[u], expect)
+        assert torch.equal(k_out[0, u].cpu(), k[0, u][torch.from_numpy(expect)])
+        assert torch.equal(v_out[0, u].cpu(), v[0, u][torch.from_numpy(expect)])
+
+
+FULL = ["llama8b-8k", "llama8b-32k", "mistral7b-16k", "llama70b-128k"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_layer_sampled_units(lib, name):
+    # the full-size layer as the benchmark runs it; the oracle checks a fixed
+    # seeded sample of units (first, last and one in the middle)
+    wl = synth.WORKLOADS[name]
+    s = synth.sensitivity_profile(wl)
+    budgets = lib.ripple_alloc_budgets(s, wl.ratio, wl.gamma, wl.global_budget)
+    layer = int(np.argmax(budgets))
+    units = [(0, 0), (wl.batch - 1, wl.n_kv_heads - 1), (wl.batch // 2, wl.n_kv_heads // 2)]
+    agree, total, _ = _check_layer(lib, wl, layer, budgets[layer], units=units, on_device=True)
+    assert agree >= 0.999 * total
+    torch.cuda.empty_cache()
