@@ -351,7 +351,11 @@ def measure_e2e(st, args, torch, tokens):
     the layer inputs and decode inputs host->device and reads the decode
     outputs back, inside the timed region."""
     wl = st.wl
-    pin = lambda t: t.to("cpu").pin_memory()
+    def pin(t):
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        return h
+
     hq = [pin(t) for t in st.q_win]
     hk = [pin(t) for t in st.k]
     hv = [pin(t) for t in st.v]
@@ -434,6 +438,22 @@ def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s):
     return step_s, sample, t_comp + t_dec
 
 
+def _decode_sampler(wl, n_keep):
+    """Seeded decode inputs of one (layer, b=0, h=0) group on the host: a cache
+    of the layer's retained length and the first decode steps' rows."""
+    from paper_2608_08684_gb300 import synth
+    G = wl.group
+
+    def get(layer, steps):
+        one = wl.replace(batch=1, n_kv_heads=1, n_q_heads=G)
+        kc, vc = synth.decode_caches(one, layer, n_keep[layer])
+        dec = [synth.decode_inputs(one, s, layers=[layer]) for s in range(steps)]
+        return (synth.to_f64(kc[0, 0]), synth.to_f64(vc[0, 0]),
+                [synth.to_f64(d[0][0, 0]) for d in dec], [synth.to_f64(d[1][0, 0, 0]) for d in dec],
+                [synth.to_f64(d[2][0, 0, 0]) for d in dec])
+    return get
+
+
 def _threads():
     try:
         import threadpoolctl
@@ -455,15 +475,7 @@ def cpu_baseline(st, target_s):
         return (synth.to_f64(st.q_win[layer][b, h * G:(h + 1) * G]), synth.to_f64(st.k[layer][b, h]),
                 synth.to_f64(st.v[layer][b, h]))
 
-    def get_decode(layer, steps):
-        n = st.n_keep[layer]
-        idx = st.idx[layer].view(wl.batch, wl.n_kv_heads, n)[0, 0].long()
-        kk = synth.to_f64(st.k[layer][0, 0].index_select(0, idx))
-        vv = synth.to_f64(st.v[layer][0, 0].index_select(0, idx))
-        qs = [synth.to_f64(st.dq[s][layer, 0, 0:G]) for s in range(steps)]
-        kns = [synth.to_f64(st.dk[s][layer, 0, 0]) for s in range(steps)]
-        vns = [synth.to_f64(st.dv[s][layer, 0, 0]) for s in range(steps)]
-        return kk, vv, qs, kns, vns
+    get_decode = _decode_sampler(wl, st.n_keep)
 
     step_s, sample, spent = oracle_sample_time(wl, get_unit, get_decode, st.budgets, st.n_keep,
                                                target_s)
@@ -500,13 +512,7 @@ def run_reference(args, rank, world):
         q, k, v = layer_tensors(layer)
         return (synth.to_f64(q[b, h * G:(h + 1) * G]), synth.to_f64(k[b, h]), synth.to_f64(v[b, h]))
 
-    def get_decode(layer, steps):
-        cap = n_keep[layer]
-        kc, vc = synth.decode_caches(wl.replace(batch=1, n_kv_heads=1), layer, cap)
-        dec = [synth.decode_inputs(wl.replace(batch=1), s, layers=[layer]) for s in range(steps)]
-        return (synth.to_f64(kc[0, 0]), synth.to_f64(vc[0, 0]),
-                [synth.to_f64(d[0][0, 0, 0:G]) for d in dec],
-                [synth.to_f64(d[1][0, 0, 0]) for d in dec], [synth.to_f64(d[2][0, 0, 0]) for d in dec])
+    get_decode = _decode_sampler(wl, n_keep)
 
     per_step = max(2.0, min(args.cpu_seconds, 120.0 / max(1, args.steps + args.warmup)))
     times, sample = [], ""
