@@ -231,6 +231,40 @@ ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
                                  void *workspace, size_t workspace_bytes,
                                  int32_t *dev_status, void *stream);
 
+/*
+ * ripple_decode_attn_noalloc -- ripple_decode_attn for callers that cannot
+ * allocate device memory. The paper has no counterpart; this is a deployment
+ * variant.
+ *
+ * Some callers have no way to obtain scratch memory on the device where they
+ * call a decode step: a plugin inside a host program that owns all device
+ * memory through its own pool and only hands over the input and output
+ * tensors, or a fixed-footprint server that reserves every byte at start-up.
+ * This entry point takes no workspace: the split-K partials of the step live
+ * in a library-owned array of RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES bytes in
+ * device global memory, which every GPU that loads the library keeps until the
+ * process exits. The caller still passes all inputs and outputs, with the
+ * meaning, layout and errors of ripple_decode_attn.
+ *
+ * - Allocates nothing: no cudaMalloc/cudaFree or allocating library call.
+ * - The first call on a device looks up the array's device address on that
+ *   device (once per device, with it current); make that first call before
+ *   any stream capture begins.
+ * - Returns RIPPLE_EWORKSPACE, before enqueuing anything, when the step needs
+ *   more partials than the array holds (ripple_decode_workspace_bytes(desc,
+ *   caps) - 256 > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
+ * - Every call on a device shares the one array, and each call overwrites
+ *   what the previous call left there (no part of it needs to start at zero).
+ *   Calls that may overlap on the GPU (different streams without ordering)
+ *   race on it; order them, e.g. by issuing them on one stream.
+ */
+#define RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
+ripple_status ripple_decode_attn_noalloc(const ripple_decode_desc *desc, const void *q,
+                                         const void *k_new, const void *v_new,
+                                         void *const *k_caches_host, void *const *v_caches_host,
+                                         const int32_t *caps_host, int32_t *lens, float *out,
+                                         int32_t *dev_status, void *stream);
+
 /* Number of kernels this library has launched in this process so far
  * (host-side count of launch calls; for benchmarks and launch accounting). */
 uint64_t ripple_kernel_launches(void);

@@ -8,6 +8,8 @@
 // partials in a fixed order (deterministic) and advances the lengths.
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -294,6 +296,99 @@ extern "C" ripple_status ripple_decode_attn(const ripple_decode_desc *desc, cons
   p.status = dev_status;
   const size_t per = (size_t)p.total_items * p.G;
   p.ws_m = (float *)workspace;
+  p.ws_l = p.ws_m + per;
+  p.ws_o = p.ws_l + per;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e;
+  if (desc->dtype == RIPPLE_F32)
+    e = p.D == 64 ? launch_d<float, 64>(p, st) : launch_d<float, 128>(p, st);
+  else
+    e = p.D == 64 ? launch_d<__nv_bfloat16, 64>(p, st) : launch_d<__nv_bfloat16, 128>(p, st);
+  return e == cudaSuccess ? RIPPLE_OK : RIPPLE_ECUDA;
+}
+
+// ---------------------------------------------------------------------------
+// Decode for callers that cannot allocate device memory (no paper counterpart).
+//
+// A plugin inside a host program that owns all device memory through its own
+// pool, or a fixed-footprint server that reserves every byte at start-up, may
+// have no way to hand this library a scratch buffer. For those callers the
+// split-K partials of a step live in the file-scope device array below
+// instead of a caller workspace. Every GPU that loads the library keeps it
+// until the process exits; all calls on a device share it and overwrite what
+// the previous call left (the partials are fully rewritten by every step, so
+// nothing needs clearing); calls that overlap on the GPU race on it.
+
+static __device__ __align__(256) float
+    g_decode_scratch[RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES / sizeof(float)];
+
+namespace {
+
+constexpr int kMaxDevices = 256;
+std::mutex g_scratch_mutex;
+float *g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_decode_scratch on the current device. In host code the
+// array's name is only a host-side handle, so the address is looked up once
+// per device (with that device current) and cached.
+ripple_status scratch_on_current_device(float **out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RIPPLE_ECUDA;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (g_scratch_addr[dev] == nullptr) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_decode_scratch) != cudaSuccess || ptr == nullptr)
+      return RIPPLE_ECUDA;
+    g_scratch_addr[dev] = (float *)ptr;
+  }
+  *out = g_scratch_addr[dev];
+  return RIPPLE_OK;
+}
+
+}  // namespace
+
+extern "C" ripple_status ripple_decode_attn_noalloc(const ripple_decode_desc *desc, const void *q,
+                                                    const void *k_new, const void *v_new,
+                                                    void *const *k_caches_host,
+                                                    void *const *v_caches_host,
+                                                    const int32_t *caps_host, int32_t *lens,
+                                                    float *out, int32_t *dev_status,
+                                                    void *stream) {
+  if (!desc_ok(desc)) return RIPPLE_EINVAL;
+  if (!q || !k_new || !v_new || !k_caches_host || !v_caches_host || !caps_host || !lens || !out)
+    return RIPPLE_EINVAL;
+  const int L = desc->n_layers;
+  auto aligned = [](const void *ptr) { return ((uintptr_t)ptr & 15u) == 0; };
+  if (!aligned(q) || !aligned(k_new) || !aligned(v_new) || !aligned(out)) return RIPPLE_EINVAL;
+  DecodeParams p;
+  for (int l = 0; l < L; ++l) {
+    if (!k_caches_host[l] || !v_caches_host[l]) return RIPPLE_EINVAL;
+    if (!aligned(k_caches_host[l]) || !aligned(v_caches_host[l])) return RIPPLE_EINVAL;
+    p.kc[l] = k_caches_host[l];
+    p.vc[l] = v_caches_host[l];
+  }
+  size_t f;
+  if (!plan(desc, caps_host, &p, &f)) return RIPPLE_EINVAL;
+  if (f * sizeof(float) > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES) return RIPPLE_EWORKSPACE;
+  float *scratch = nullptr;
+  const ripple_status s = scratch_on_current_device(&scratch);
+  if (s != RIPPLE_OK) return s;
+  p.L = L;
+  p.B = desc->batch;
+  p.Hq = desc->n_q_heads;
+  p.Hkv = desc->n_kv_heads;
+  p.G = p.Hq / p.Hkv;
+  p.D = desc->head_dim;
+  const float scale = desc->scale > 0.f ? desc->scale : 1.0f / sqrtf((float)p.D);
+  p.scale2 = scale * kLog2e;
+  p.q = q;
+  p.k_new = k_new;
+  p.v_new = v_new;
+  p.lens = lens;
+  p.out = out;
+  p.status = dev_status;
+  const size_t per = (size_t)p.total_items * p.G;
+  p.ws_m = scratch;
   p.ws_l = p.ws_m + per;
   p.ws_o = p.ws_l + per;
   cudaStream_t st = (cudaStream_t)stream;

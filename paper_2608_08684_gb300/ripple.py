@@ -71,6 +71,10 @@ _lib.ripple_decode_attn.argtypes = [ctypes.POINTER(DecodeDesc), _p, _p, _p, ctyp
                                     ctypes.POINTER(_p), ctypes.POINTER(_i32), _p, _p, _p, _sz, _p,
                                     _p]
 _lib.ripple_decode_attn.restype = _i32
+_lib.ripple_decode_attn_noalloc.argtypes = [ctypes.POINTER(DecodeDesc), _p, _p, _p,
+                                            ctypes.POINTER(_p), ctypes.POINTER(_p),
+                                            ctypes.POINTER(_i32), _p, _p, _p, _p]
+_lib.ripple_decode_attn_noalloc.restype = _i32
 _lib.ripple_kernel_launches.argtypes = []
 _lib.ripple_kernel_launches.restype = ctypes.c_uint64
 _lib.ripple_status_string.argtypes = [_i32]
@@ -197,6 +201,23 @@ def ripple_decode_attn(desc: DecodeDesc, q, k_new, v_new, tables: DecodeTables, 
                                    _ptr(workspace), workspace.numel() * workspace.element_size(),
                                    _ptr(dev_status), _stream(stream)),
            "ripple_decode_attn")
+
+
+NOALLOC_SCRATCH_BYTES = 8 << 20
+
+
+def ripple_decode_attn_noalloc(desc: DecodeDesc, q, k_new, v_new, tables: DecodeTables, lens,
+                               out, dev_status=None, stream=None):
+    """ripple_decode_attn without a workspace argument, for callers that cannot
+    allocate device memory (for instance a plugin whose host owns every device
+    buffer and only passes tensors in and out). The split-K partials live in
+    the library's own fixed device array of NOALLOC_SCRATCH_BYTES; steps that
+    need more raise RippleError(EWORKSPACE). Calls overlapping on the GPU race
+    on that array."""
+    _check(_lib.ripple_decode_attn_noalloc(ctypes.byref(desc), _ptr(q), _ptr(k_new), _ptr(v_new),
+                                           tables.k, tables.v, tables.caps, _ptr(lens),
+                                           _ptr(out), _ptr(dev_status), _stream(stream)),
+           "ripple_decode_attn_noalloc")
 
 
 def ripple_kernel_launches() -> int:
