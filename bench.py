@@ -54,7 +54,86 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU seconds of the oracle sample")
+    ap.add_argument("--case", choices=["compress", "decode"], default=None,
+                    help="time one entry point alone (one layer / one decode step), e.g. "
+                         "as a small ncu target; prints one JSON line")
+    ap.add_argument("--repeat", type=int, default=10, help="calls timed in --case mode")
     return ap.parse_args()
+
+
+def run_case(args):
+    """Single-entry-point timing: compression of the workload's largest-budget
+    layer, or one decode step over every layer's ragged cache (seeded caches
+    at the RippleKV sizes). Inputs stay within a few GB of device memory."""
+    import torch
+
+    from paper_2608_08684_gb300 import build as _build
+    from paper_2608_08684_gb300 import synth
+    _build.build_library()
+    from paper_2608_08684_gb300 import ripple as R
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    wl = synth.WORKLOADS[args.workload]
+    L, B, Hq, Hkv, d, e = (wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim,
+                           wl.elem_bytes)
+    budgets = R.ripple_alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
+                                     wl.global_budget)
+    n_keep = [R.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    times = []
+    if args.case == "compress":
+        layer = max(range(L), key=lambda i: budgets[i])
+        q_win = synth.layer_window_queries(wl, layer, dev)
+        k = synth.layer_keys(wl, layer, dev)
+        v = synth.layer_values(wl, layer, dev)
+        desc = R.layer_desc(B, Hq, Hkv, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                            wl.torch_dtype)
+        n = n_keep[layer]
+        ws = torch.empty(R.ripple_compress_workspace_bytes(desc), dtype=torch.uint8, device=dev)
+        k_out = torch.empty(B, Hkv, n, d, dtype=wl.torch_dtype, device=dev)
+        v_out = torch.empty_like(k_out)
+        idx = torch.empty(B * Hkv * n, dtype=torch.int32, device=dev)
+        nbytes = B * Hkv * d * e * (wl.seq_len + 3 * n) + B * Hq * wl.window * d * e
+        for i in range(args.repeat + 2):
+            a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            R.ripple_compress_layer(desc, budgets[layer], q_win, k, v, k_out, v_out, idx, ws,
+                                    dev_status=status)
+            b_.record()
+            if i >= 2:
+                times.append((a, b_))
+        what = f"compress layer {layer} (budget {budgets[layer]}, n {n})"
+    else:
+        caps = [n + 1 for n in n_keep]
+        kc, vc = zip(*[synth.decode_caches(wl, i, caps[i], dev) for i in range(L)])
+        tables = R.DecodeTables(list(kc), list(vc))
+        ddesc = R.decode_desc(L, B, Hq, Hkv, d, wl.torch_dtype)
+        dws = torch.empty(R.ripple_decode_workspace_bytes(ddesc, caps), dtype=torch.uint8,
+                          device=dev)
+        lens0 = torch.tensor(n_keep, dtype=torch.int32, device=dev)
+        lens = lens0.clone()
+        q, kn, vn = synth.decode_inputs(wl, 0, dev)
+        out = torch.empty(L, B, Hq, d, device=dev)
+        nbytes = (sum(B * Hkv * 2 * (n + 1) * d * e for n in n_keep)
+                  + L * B * Hq * d * (e + 4) + L * B * Hkv * d * e * 4)
+        for i in range(args.repeat + 2):
+            lens.copy_(lens0)
+            a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            R.ripple_decode_attn(ddesc, q, kn, vn, tables, lens, out, dws, dev_status=status)
+            b_.record()
+            if i >= 2:
+                times.append((a, b_))
+        what = f"decode step over {L} layers, lens {min(n_keep)}..{max(n_keep)}"
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0, int(status.item())
+    ms = statistics.mean(a.elapsed_time(b) for a, b in times)
+    hbm, src = measured_peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    print(json.dumps({"case": args.case, "workload": wl.name, "what": what, "calls": len(times),
+                      "ms_per_call": round(ms, 5), "bytes_per_call": nbytes,
+                      "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
+                      "peak_source": src}), flush=True)
 
 
 def measured_peaks():
@@ -540,7 +619,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", str(args.gpus if args.gpus == 1 else 1)))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
-    if args.impl == "reference":
+    if args.case:
+        run_case(args)
+    elif args.impl == "reference":
         run_reference(args, rank, world)
     else:
         run_ours(args, rank, world, local_rank)

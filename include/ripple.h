@@ -251,10 +251,11 @@ ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
  *   device (once per device, with it current); make that first call before
  *   any stream capture begins.
  * - Returns RIPPLE_EWORKSPACE, before enqueuing anything, when the step needs
- *   more partials than the array holds (ripple_decode_workspace_bytes(desc,
- *   caps) - 256 > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
- * - Every call on a device shares the one array, and each call overwrites
- *   what the previous call left there (no part of it needs to start at zero).
+ *   more scratch than the array holds (ripple_decode_workspace_bytes(desc,
+ *   caps) > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
+ * - Every call on a device shares the one array. Each call clears the
+ *   counters it uses at its start (a memset enqueued on `stream`) and rewrites
+ *   every partial it reads, so nothing carries over from the previous call.
  *   Calls that may overlap on the GPU (different streams without ordering)
  *   race on it; order them, e.g. by issuing them on one stream.
  */

@@ -56,6 +56,13 @@ __device__ __forceinline__ float fast_exp2(float x) {
   return y;
 }
 
+// Named barrier over `threads` threads (a multiple of 32); the warp converges
+// first because bar.sync is warp-aligned.
+__device__ __forceinline__ void named_bar_sync(int id, int threads) {
+  __syncwarp();
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
 // First error code wins.
 __device__ __forceinline__ void report(int32_t *status, int32_t code) {
   if (status != nullptr) atomicCAS(status, 0, code);

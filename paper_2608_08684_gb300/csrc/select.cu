@@ -109,9 +109,14 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
     const uint32_t dmask = (1u << widths[round]) - 1u;
     for (int i = tid; i < kBins; i += kThreads) hist[i] = 0;
     __syncthreads();
-    for (int t = tid; t < P; t += kThreads) {
-      const uint32_t u = keys[t];
-      if ((u & mask) == prefix) atomicAdd(&hist[(u >> shift) & dmask], 1u);
+    // Scores cluster in few bins: lanes with the same bin add once per warp.
+    for (int base = 0; base < P; base += kThreads) {
+      const int t = base + tid;
+      const uint32_t u = t < P ? keys[t] : 0u;
+      const bool hit = t < P && (u & mask) == prefix;
+      const uint32_t bin = hit ? (u >> shift) & dmask : 0xffffffffu;
+      const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+      if (hit && (threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
     }
     __syncthreads();
     // Thread j owns digits 2047-2j and 2046-2j (descending).
