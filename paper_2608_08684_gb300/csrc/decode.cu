@@ -6,9 +6,10 @@
 // of one (layer, batch row, KV head) group's cache rows; items are fetched
 // with an atomic counter, layers with the longest caches first (longest-
 // processing-time order). The producer warp stages each sub-chunk's K and V
-// rows in shared memory with bulk-async (TMA engine) copies, double-buffered,
-// and writes the new token's rows into the stage (and appends them to the
-// cache). Every compute warp owns CR/16 rows of each sub-chunk and keeps its
+// rows in shared memory with bulk-async (TMA engine) copies, two stages
+// deep plus an L2 prefetch further ahead, and writes the new token's rows into
+// the stage (and appends them to the cache). Every compute warp owns CR/16
+// rows of each sub-chunk and keeps its
 // own online-softmax state, so no block-wide barrier is needed per sub-chunk
 // (stages are released through mbarriers):
 //   scores  q_g . k_row * scale * log2(e): S lanes per row, the query slice in
@@ -34,8 +35,9 @@ constexpr int kWarps = 16;                    // compute warps
 constexpr int kThreads = (kWarps + 1) * 32;   // + one producer warp
 constexpr int kStageBytes = 32768;            // K (or V) bytes of one sub-chunk
 constexpr int kStages = 2;
-constexpr int kItemSub = 4;                   // sub-chunks per work item
+constexpr int kItemSub = 16;                  // sub-chunks per work item (merges are costly)
 constexpr int kItemSlots = 4;
+constexpr int kPrefetchAhead = 2;             // sub-chunks prefetched into L2 past the stages
 
 template <typename Tin, int D, int G>
 struct DecCfg {
@@ -154,6 +156,31 @@ __device__ __forceinline__ void load_pairs(const float *p, float2 (&o)[NP]) {
   }
 }
 
+// L2 prefetch of one sub-chunk's cache rows (K and V, rows before the new
+// token); `sub` may run past the item's end into the following item.
+template <typename Tin, int D, int G>
+__device__ __forceinline__ void prefetch_sub(const DecParams &p, const DecSmem<Tin, D, G> &s,
+                                             int total, int it, int nxt, int sub) {
+  using C = DecCfg<Tin, D, G>;
+  if (it >= total) return;
+  ItemInfo f = item_info(p, s, it);
+  int nsub = f.full ? 0 : (f.rows + C::CR - 1) / C::CR;
+  if (sub >= nsub) {
+    sub -= nsub;
+    if (nxt >= total) return;
+    f = item_info(p, s, nxt);
+    nsub = f.full ? 0 : (f.rows + C::CR - 1) / C::CR;
+    if (sub >= nsub) return;
+  }
+  const int rs = f.r0 + sub * C::CR;
+  const int re = min(rs + C::CR, f.len);
+  if (re <= rs) return;
+  const size_t off = ((size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer] + rs) * C::ROW_BYTES;
+  const uint32_t bytes = (uint32_t)(re - rs) * C::ROW_BYTES;
+  bulk_prefetch_l2((const uint8_t *)p.kc[f.layer] + off, bytes);
+  bulk_prefetch_l2((const uint8_t *)p.vc[f.layer] + off, bytes);
+}
+
 template <int G>
 __device__ __forceinline__ void load_probs(const float *src, float (&pr)[G]) {
   if constexpr (G % 4 == 0) {
@@ -214,7 +241,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     int icount = 0;
     uint32_t j = 0;
     int it = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
+    int nxt = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
     it = __shfl_sync(0xffffffffu, it, 0);
+    nxt = __shfl_sync(0xffffffffu, nxt, 0);
     for (;;) {
       const int slot = icount % kItemSlots;
       mbar_wait(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, p.status);
@@ -225,7 +254,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       }
       ++icount;
       if (it >= total) break;
-      int nxt = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
+      // The first sub-chunks of the very first item get an L2 prefetch too.
+      if (lane == 0 && icount == 1)
+        for (int k = 0; k < kPrefetchAhead; ++k) prefetch_sub(p, s, total, it, nxt, k);
+      int nxt2 = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
       const ItemInfo f = item_info(p, s, it);
       if (!f.full) {
         const int nsub = (f.rows + C::CR - 1) / C::CR;
@@ -263,10 +295,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
             } else {
               mbar_arrive(&s.full[stage]);
             }
+            // Keep kPrefetchAhead more sub-chunks on their way into L2.
+            prefetch_sub(p, s, total, it, nxt, sub + kPrefetchAhead);
           }
         }
       }
-      it = __shfl_sync(0xffffffffu, nxt, 0);
+      it = nxt;
+      nxt = __shfl_sync(0xffffffffu, nxt2, 0);
     }
   } else {
     // ------------------------------------------------ compute warps
@@ -297,13 +332,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
 #pragma unroll
         for (int g = 0; g < G; ++g)
 #pragma unroll
-          for (int k = 0; k < C::PPL; ++k)
+          for (int k = 0; k < C::PPL; ++k) {
+            float2 t[C::PE / 2];
+            load_pairs<C::PE / 2>(qg + g * D + (slot_l + k * C::S) * C::PE, t);
 #pragma unroll
-            for (int e = 0; e < C::PE; e += 2) {
-              const int dim = (slot_l + k * C::S) * C::PE + e;
-              q2[g][(k * C::PE + e) / 2] = make_float2(to_f32(qg[g * D + dim]) * p.scale2,
-                                                       to_f32(qg[g * D + dim + 1]) * p.scale2);
-            }
+            for (int e = 0; e < C::PE / 2; ++e)
+              q2[g][k * C::PE / 2 + e] = make_float2(t[e].x * p.scale2, t[e].y * p.scale2);
+          }
       }
       float2 acc[G][C::DV / 2];
 #pragma unroll
@@ -407,7 +442,9 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
               acc[g][e].y *= a[g];
             }
           const int rmax = min(C::RPW, nrows - rw0);
-          for (int r = 0; r < rmax; ++r) {
+#pragma unroll
+          for (int r = 0; r < C::RPW; ++r) {
+            if (r >= rmax) break;
             float pr[G];
             load_probs<G>(s.pw[warp][r], pr);
             float2 vp[C::DV / 2];

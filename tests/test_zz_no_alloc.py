@@ -61,7 +61,7 @@ def test_noalloc_rejects_steps_beyond_its_scratch(lib):
     # caps whose partials exceed the fixed array are refused before any launch
     wl = synth.WORKLOADS["tiny"].replace(n_layers=1, batch=64, n_q_heads=64, n_kv_heads=8,
                                          head_dim=128, dtype="bf16")
-    caps = [4096]
+    caps = [32768]
     desc = lib.decode_desc(1, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.torch_dtype)
     assert lib.ripple_decode_workspace_bytes(desc, caps) > lib.NOALLOC_SCRATCH_BYTES
     # the request is refused on the host from desc and caps alone, so small
