@@ -29,7 +29,8 @@ CompressWs carve_compress_ws(const LayerGeom &g, void *base) {
     off += round_up(bytes);
     return r;
   };
-  w.row_partial = (float2 *)take(sizeof(float2) * g.units * n_chunks * g.R);
+  // two partials per chunk: the tensor-core path keeps one per epilogue warpgroup
+  w.row_partial = (float2 *)take(sizeof(float2) * g.units * n_chunks * 2 * g.R);
   w.row_lognorm = (float *)take(sizeof(float) * g.units * g.R);
   w.votes = (float *)take(sizeof(float) * g.units * (size_t)g.P);
   w.keys = (uint32_t *)take(g.P > kSelectSmemKeys ? sizeof(uint32_t) * g.units * (size_t)g.P : 0);

@@ -27,7 +27,7 @@ constexpr int kSelectSmemKeys = 48 * 1024;  // prefix lengths up to this keep ke
 
 // Workspace carve-up of one compression call.
 struct CompressWs {
-  float2 *row_partial;  // [units][n_chunks][R] (max, sum) in the log2 domain
+  float2 *row_partial;  // [units][n_chunks][2][R] (max, sum) in the log2 domain
   float *row_lognorm;   // [units][R] max + log2(sum), log2 domain
   float *votes;         // [units][P] unpooled votes (when scores_out is NULL)
   uint32_t *keys;       // [units][P] pooled-score sort keys (long prefixes only)

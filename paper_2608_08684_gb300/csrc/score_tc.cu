@@ -5,24 +5,30 @@
 // causal inside the window, softmax per row over all visible keys, vote of a
 // prefix key = sum over rows of its probability.
 //
-// One persistent launch per layer (grid = SM count, one CTA per SM) does both
-// passes over every unit (b, h) of the layer:
-//   pass 1 item (unit, chunk): per window row, (max, sum of exp) over the
-//     chunk's key tiles -> partial[unit][chunk][row]; the CTA finishing the
-//     unit's last chunk merges them into lognorm[unit][row] = max + log2(sum)
-//     and raises ready[unit];
-//   pass 2 item (unit, chunk): per prefix key of the chunk, vote = sum over
-//     rows of exp2(x * scale * log2e - lognorm[row]), after ready[unit].
-// Items are fetched dynamically in a list ordered group by group,
-// P1(0) P1(1) P2(0) P1(2) P2(1) ..., with groups of units sized so that a
-// unit's keys are still in L2 when pass 2 re-reads them.
+// One launch per layer, one persistent CTA per SM, co-resident (cooperative
+// launch). A unit (b, h) is cut into items of `tpi` key tiles; item i belongs
+// to CTA i mod grid, so every unit is spread over many CTAs that work on it at
+// the same time. Each CTA runs its items in the order
+//     P1(a0) P1(a1) P2(a0) P1(a2) P2(a1) ...
+//   pass 1 of an item: per window row, (max, sum of exp) over the item's key
+//     tiles -> partial[unit][item][row] (the publisher warp combines the two
+//     epilogue warpgroups' statistics); it counts the unit's finished items
+//     and the last one merges them into
+//     lognorm[unit][row] = max + log2(sum) and raises ready[unit];
+//   pass 2 of an item: per prefix key, vote = sum over rows of
+//     exp2(x * scale * log2e - lognorm[row]), once ready[unit] is up.
+// An item's keys are read again one item later, so the second read is served
+// from L2 (about two items per SM are in flight). A pass-2 wait only depends
+// on first passes of strictly earlier units as long as a unit has at most
+// twice as many items as there are CTAs, so with every CTA resident the
+// schedule cannot deadlock.
 //
-// Warp roles (320 threads): warp 0 = TMA producer, warp 1 = MMA issuer and
-// TMEM owner, warps 2-9 = two epilogue warpgroups taking alternate key tiles.
-// Pass 1 computes D[row][key] (A = window queries, B = key tile, M = 128 per
-// row block); pass 2 computes D[key][row] (A = key tile, B = window queries,
-// N = G*w), so that each epilogue thread owns one row (pass 1) or one key
-// (pass 2) and every reduction is thread-local.
+// Warp roles (352 threads): warp 0 = TMA producers (keys, queries), warp 1 = MMA issuer and
+// TMEM owner, warps 2-9 = two epilogue warpgroups taking alternate key tiles,
+// warp 10 = publisher of pass-1 results. Pass 1 computes D[row][key]
+// (A = window queries, B = key tile); pass 2 computes D[key][row] (A = key
+// tile, B = window queries), so each epilogue thread owns one row (pass 1) or
+// one key (pass 2) and every reduction is thread-local.
 // Every wait is bounded: on timeout the CTA raises RIPPLE_ETIMEOUT, all roles
 // leave their loops, and TMEM is released.
 #include <cuda.h>
@@ -37,8 +43,9 @@ namespace {
 constexpr int kTile = 128;                      // keys per tile
 constexpr int kHalfBytes = kTile * 64 * 2;      // 64 bf16 columns of 128 rows: 16 KB
 constexpr int kTileBytes = 2 * kHalfBytes;      // one 128 x 128 bf16 tile
-constexpr int kThreads = 320;
-constexpr int kItemSlots = 4;
+constexpr int kThreads = 352;
+constexpr int kPubSlots = 2;
+constexpr int kMinTilesPerItem = 8;
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 // ------------------------------------------------------------ PTX wrappers
@@ -52,13 +59,26 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
       : "memory");
 }
 
+// 3-D tile load with an L2 cache policy (evict_last keeps an item's keys for
+// its second pass, evict_first lets the second pass's reads go).
 __device__ __forceinline__ void tma_load_3d(void *dst, const CUtensorMap *map, int x, int y, int z,
-                                            uint64_t *bar) {
+                                            uint64_t *bar, uint64_t policy) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
-      "l"((uint64_t)map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(dst)),
+      "l"((uint64_t)map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
       : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
 }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst, uint32_t ncols) {
@@ -117,12 +137,6 @@ __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Named barrier; the warp is converged first (bar.sync is warp-aligned).
-__device__ __forceinline__ void named_bar(int id, int threads) {
-  __syncwarp();
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
-}
-
 __device__ __forceinline__ int ld_acquire(const int *p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -153,46 +167,36 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
 
 struct TcParams {
   int units, T, P, W, Hq, Hkv, G;
-  int n_tiles1, n_tiles2, chunk, n_ch1, n_ch2, group_units, n_groups, n_items;
+  int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys)
+  int tpi, n_ch;           // key tiles per item, items per unit
+  int total_items;
   float scale2;
-  float2 *partial;  // [units][n_ch1][R]
+  float2 *partial;  // [units][n_ch][R] (max, sum) per item and row, log2 domain
   float *lognorm;   // [units][R]
   float *votes;     // [units][P]
-  int *ctrl;        // [0] item counter; [32 + u] pass-1 chunks done; [32 + units + u] ready
+  int *ctrl;        // [u] items of unit u published; [units + u] row statistics ready
   int32_t *status;
 };
 
-struct Item {
-  int pass, unit, chunk;  // pass 0 marks the end of the work
+struct ItemRef {
+  int unit, chunk;
 };
 
-__device__ Item decode_item(const TcParams &p, int idx) {
-  if (idx >= p.n_items) return {0, 0, 0};
-  for (int k = 0; k < 2 * p.n_groups; ++k) {
-    int pass, g;
-    if (k == 0) {
-      pass = 1; g = 0;
-    } else if (k == 2 * p.n_groups - 1) {
-      pass = 2; g = p.n_groups - 1;
-    } else if (k & 1) {
-      pass = 1; g = (k + 1) / 2;
-    } else {
-      pass = 2; g = k / 2 - 1;
-    }
-    const int u0 = g * p.group_units;
-    const int ug = min(p.group_units, p.units - u0);
-    const int nch = pass == 1 ? p.n_ch1 : p.n_ch2;
-    const int sz = ug * nch;
-    if (idx < sz) return {pass, u0 + idx / nch, idx % nch};
-    idx -= sz;
-  }
-  return {0, 0, 0};
+// The k-th item of this CTA.
+__device__ __forceinline__ ItemRef item_of(const TcParams &p, int k) {
+  const int i = (int)blockIdx.x + k * (int)gridDim.x;
+  return {i / p.n_ch, i % p.n_ch};
 }
 
-__device__ __forceinline__ void item_tiles(const TcParams &p, const Item &it, int &t0, int &t1) {
-  const int n = it.pass == 1 ? p.n_tiles1 : p.n_tiles2;
-  t0 = it.chunk * p.chunk;
-  t1 = min(n, t0 + p.chunk);
+__device__ __forceinline__ int items_of_cta(const TcParams &p) {
+  const int b = (int)blockIdx.x;
+  return b < p.total_items ? (p.total_items - 1 - b) / (int)gridDim.x + 1 : 0;
+}
+
+__device__ __forceinline__ void tiles_of(const TcParams &p, const ItemRef &it, int pass, int &t0,
+                                         int &t1) {
+  t0 = it.chunk * p.tpi;
+  t1 = min(pass == 1 ? p.n_tiles1 : p.n_tiles2, t0 + p.tpi);
 }
 
 // ------------------------------------------------------------ shared memory
@@ -200,8 +204,10 @@ __device__ __forceinline__ void item_tiles(const TcParams &p, const Item &it, in
 template <int NR>
 struct Cfg {
   static constexpr int R = 128 * NR;             // window rows
-  static constexpr int NK = NR == 1 ? 4 : 2;     // key-tile stages
-  static constexpr int NQ = 2;                   // query buffers
+  static constexpr int NK = NR == 1 ? 3 : 2;     // key-tile stages
+  // Query buffers: two items are in flight (pass 1 of one, pass 2 of the
+  // previous); a third lets the next item's queries load ahead.
+  static constexpr int NQ = NR == 1 ? 3 : 2;
   static constexpr int NA = NR == 1 ? 4 : 2;     // TMEM accumulator stages
   static constexpr int ACC_COLS = 128 * NR;      // TMEM columns per stage
   static constexpr int QBYTES = R * 256;         // R rows x 128 bf16
@@ -211,18 +217,15 @@ struct Cfg {
 };
 
 struct Misc {
-  uint64_t k_full[4], k_empty[4], q_full[2], q_empty[2], acc_full[4], acc_empty[4], mma_done;
-  uint64_t item_full[kItemSlots], item_empty[kItemSlots];
-  Item items[kItemSlots];
+  uint64_t k_full[4], k_empty[4], q_full[3], q_empty[3], acc_full[4], acc_empty[4], mma_done;
+  uint64_t pub_full[kPubSlots], pub_empty[kPubSlots];
   uint32_t tmem_base;
   int abort_flag;
-  int last_flag;
-  alignas(16) float off[2][256];  // per-warpgroup row offsets of a pass-2 item (read as float4)
-  alignas(16) float2 xch[256];    // warpgroup 1 -> 0 exchange of pass-1 row stats
+  alignas(16) float off[2][256];  // per-warpgroup row log-normalisers of a pass-2 item
+  float2 pstat[kPubSlots][2][256];  // pass-1 row statistics per slot and warpgroup
 };
 
-static_assert(offsetof(Misc, off) % 16 == 0 && offsetof(Misc, xch) % 16 == 0,
-              "vector-accessed shared arrays must be 16-byte aligned");
+static_assert(offsetof(Misc, off) % 16 == 0, "float4-read shared arrays are 16-byte aligned");
 
 template <int NR>
 constexpr int smem_bytes() {
@@ -245,8 +248,8 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *m
   }
 }
 
-// Warp-uniform variant for the epilogue warps: all lanes wait, the warp then
-// agrees on the outcome (and is converged for the .sync.aligned TMEM loads).
+// Warp-uniform variant: all lanes wait, the warp then agrees on the outcome
+// (and is converged for the .sync.aligned TMEM loads that follow).
 __device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Misc *ms,
                                           int32_t *status) {
   const bool ok = wait_bar(bar, parity, ms, status);
@@ -288,6 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t *qbufs = smem + C::OFF_Q;
   Misc *ms = (Misc *)(smem + C::OFF_MISC);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = items_of_cta(p);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < C::NK; ++i) {
@@ -302,9 +306,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->acc_full[i], 1);
       mbar_init(&ms->acc_empty[i], 4);
     }
-    for (int i = 0; i < kItemSlots; ++i) {
-      mbar_init(&ms->item_full[i], 1);
-      mbar_init(&ms->item_empty[i], 1 + 8);
+    for (int i = 0; i < kPubSlots; ++i) {
+      mbar_init(&ms->pub_full[i], 8);
+      mbar_init(&ms->pub_empty[i], 1);
     }
     mbar_init(&ms->mma_done, 1);
     ms->abort_flag = 0;
@@ -319,24 +323,50 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = ms->tmem_base;
 
+  // Every role walks the same sequence: for k = 0..n, P1(item k) if k < n,
+  // then P2(item k - 1) if k >= 1.
   if (warp == 0) {
-    // ------------------------------------------------ TMA producer
+    // ------------------------------------------------ TMA producers
+    // Lane 0 streams key tiles through the ring; lane 1 loads each item's
+    // window queries as soon as a query buffer is free, so that the key
+    // stream never waits for a query load.
     if (lane == 0) {
-      int kcount = 0, qcount = 0, icount = 0;
-      int next = atomicAdd(&p.ctrl[0], 1);
-      for (;;) {
-        const Item it = decode_item(p, next);
-        if (it.pass) next = atomicAdd(&p.ctrl[0], 1);
-        const int slot = icount % kItemSlots;
-        if (!wait_bar(&ms->item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, ms, p.status)) break;
-        ms->items[slot] = it;
-        mbar_arrive(&ms->item_full[slot]);
-        ++icount;
-        if (!it.pass) break;
+      int kcount = 0;
+      const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
+      bool ok = true;
+      for (int k = 0; k <= n && ok; ++k) {
+        for (int pass = 1; pass <= 2 && ok; ++pass) {
+          if ((pass == 1 && k >= n) || (pass == 2 && k < 1)) continue;
+          const ItemRef it = item_of(p, pass == 1 ? k : k - 1);
+          int t0, t1;
+          tiles_of(p, it, pass, t0, t1);
+          for (int t = t0; t < t1; ++t) {
+            const int ks = kcount % C::NK;
+            if (!wait_bar(&ms->k_empty[ks], ((kcount / C::NK) & 1) ^ 1, ms, p.status)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
+            uint8_t *kb = ktiles + ks * kTileBytes;
+            const uint64_t pol = pass == 1 ? keep : drop;
+            tma_load_3d(kb, &kmap, 0, t * kTile, it.unit, &ms->k_full[ks], pol);
+            tma_load_3d(kb + kHalfBytes, &kmap, 64, t * kTile, it.unit, &ms->k_full[ks], pol);
+            ++kcount;
+          }
+        }
+      }
+      // Let every issued copy land before the CTA can exit (matters only after
+      // an abort; in normal operation every stage was already consumed).
+      for (int j = max(0, kcount - C::NK); j < kcount; ++j)
+        mbar_wait(&ms->k_full[j % C::NK], (j / C::NK) & 1, nullptr, kWaitCycles / 4);
+    } else if (lane == 1) {
+      int qcount = 0;
+      for (int k = 0; k < n; ++k) {
+        const ItemRef it = item_of(p, k);
         const int b = it.unit / p.Hkv, h = it.unit % p.Hkv;
         const int qrow0 = (b * p.Hq + h * p.G) * p.W;
-        const int qs = qcount % C::NQ;
-        if (!wait_bar(&ms->q_empty[qs], ((qcount / C::NQ) & 1) ^ 1, ms, p.status)) break;
+        const int qs = k % C::NQ;
+        if (!wait_bar(&ms->q_empty[qs], ((k / C::NQ) & 1) ^ 1, ms, p.status)) break;
         mbar_arrive_expect_tx(&ms->q_full[qs], C::QBYTES);
         uint8_t *qb = qbufs + qs * C::QBYTES;
         for (int half = 0; half < 2; ++half)
@@ -344,85 +374,122 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(qb + half * (NR * kHalfBytes) + nr * kHalfBytes, &qmap, half * 64,
                         qrow0 + nr * 128, &ms->q_full[qs]);
         ++qcount;
-        int t0, t1;
-        item_tiles(p, it, t0, t1);
-        bool ok = true;
-        for (int t = t0; t < t1; ++t) {
-          const int ks = kcount % C::NK;
-          if (!wait_bar(&ms->k_empty[ks], ((kcount / C::NK) & 1) ^ 1, ms, p.status)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
-          uint8_t *kb = ktiles + ks * kTileBytes;
-          tma_load_3d(kb, &kmap, 0, t * kTile, it.unit, &ms->k_full[ks]);
-          tma_load_3d(kb + kHalfBytes, &kmap, 64, t * kTile, it.unit, &ms->k_full[ks]);
-          ++kcount;
-        }
-        if (!ok) break;
       }
-      // Let every issued copy land before the CTA can exit (matters only after
-      // an abort; in normal operation every stage was already consumed).
-      for (int j = max(0, kcount - C::NK); j < kcount; ++j)
-        mbar_wait(&ms->k_full[j % C::NK], (j / C::NK) & 1, nullptr, kWaitCycles / 4);
-      for (int j = max(0, qcount - C::NQ); j < qcount; ++j)
-        mbar_wait(&ms->q_full[j % C::NQ], (j / C::NQ) & 1, nullptr, kWaitCycles / 4);
+      for (int k = max(0, qcount - C::NQ); k < qcount; ++k)
+        mbar_wait(&ms->q_full[k % C::NQ], (k / C::NQ) & 1, nullptr, kWaitCycles / 4);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int kcount = 0, qcount = 0, icount = 0, acount = 0;
+      int kcount = 0, acount = 0;
       constexpr uint32_t id1 = idesc_bf16(128, 128);
       constexpr uint32_t id2 = idesc_bf16(128, 128 * NR);
       const uint32_t kbase = smem_u32(ktiles), qbase = smem_u32(qbufs);
-      for (;;) {
-        const int slot = icount % kItemSlots;
-        if (!wait_bar(&ms->item_full[slot], (icount / kItemSlots) & 1, ms, p.status)) break;
-        const Item it = ms->items[slot];
-        mbar_arrive(&ms->item_empty[slot]);
-        ++icount;
-        if (!it.pass) break;
-        const int qs = qcount % C::NQ;
-        if (!wait_bar(&ms->q_full[qs], (qcount / C::NQ) & 1, ms, p.status)) break;
-        const uint32_t qa = qbase + qs * C::QBYTES;
-        int t0, t1;
-        item_tiles(p, it, t0, t1);
-        bool ok = true;
-        for (int t = t0; t < t1; ++t) {
-          const int ks = kcount % C::NK, as = acount % C::NA;
-          if (!wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status) ||
-              !wait_bar(&ms->acc_empty[as], ((acount / C::NA) & 1) ^ 1, ms, p.status)) {
+      bool ok = true;
+      for (int k = 0; k <= n && ok; ++k) {
+        for (int pass = 1; pass <= 2 && ok; ++pass) {
+          if ((pass == 1 && k >= n) || (pass == 2 && k < 1)) continue;
+          const int item = pass == 1 ? k : k - 1;
+          const ItemRef it = item_of(p, item);
+          const int qs = item % C::NQ;
+          if (pass == 1 && !wait_bar(&ms->q_full[qs], (item / C::NQ) & 1, ms, p.status)) {
             ok = false;
             break;
           }
-          tc_fence_after();
-          const uint32_t d = tmem + as * C::ACC_COLS;
-          const uint32_t ka = kbase + ks * kTileBytes;
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t koff = (k >> 2) * kHalfBytes + (k & 3) * 32;
-            const uint32_t qoff = (k >> 2) * (NR * kHalfBytes) + (k & 3) * 32;
-            if (it.pass == 1) {
-#pragma unroll
-              for (int nr = 0; nr < NR; ++nr)
-                mma_bf16(d + nr * 128, sw128_desc(qa + qoff + nr * kHalfBytes),
-                         sw128_desc(ka + koff), id1, k > 0);
-            } else {
-              mma_bf16(d, sw128_desc(ka + koff), sw128_desc(qa + qoff), id2, k > 0);
+          const uint32_t qa = qbase + qs * C::QBYTES;
+          int t0, t1;
+          tiles_of(p, it, pass, t0, t1);
+          for (int t = t0; t < t1; ++t) {
+            const int ks = kcount % C::NK, as = acount % C::NA;
+            if (!wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status) ||
+                !wait_bar(&ms->acc_empty[as], ((acount / C::NA) & 1) ^ 1, ms, p.status)) {
+              ok = false;
+              break;
             }
+            tc_fence_after();
+            const uint32_t d = tmem + as * C::ACC_COLS;
+            const uint32_t ka = kbase + ks * kTileBytes;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+              const uint32_t qoff = (kk >> 2) * (NR * kHalfBytes) + (kk & 3) * 32;
+              if (pass == 1) {
+#pragma unroll
+                for (int nr = 0; nr < NR; ++nr)
+                  mma_bf16(d + nr * 128, sw128_desc(qa + qoff + nr * kHalfBytes),
+                           sw128_desc(ka + koff), id1, kk > 0);
+              } else {
+                mma_bf16(d, sw128_desc(ka + koff), sw128_desc(qa + qoff), id2, kk > 0);
+              }
+            }
+            mma_commit(&ms->k_empty[ks]);
+            mma_commit(&ms->acc_full[as]);
+            ++kcount;
+            ++acount;
           }
-          mma_commit(&ms->k_empty[ks]);
-          mma_commit(&ms->acc_full[as]);
-          ++kcount;
-          ++acount;
+          if (ok && pass == 2) mma_commit(&ms->q_empty[qs]);  // the item is done with its queries
         }
-        if (!ok) break;
-        mma_commit(&ms->q_empty[qs]);
-        ++qcount;
       }
       // All issued MMAs complete before TMEM is released.
       mma_commit(&ms->mma_done);
       mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
+    }
+  } else if (warp == 10) {
+    // ------------------------------------------------ publisher of pass-1 results
+    constexpr int RJ = C::R / 32;   // rows per lane
+    constexpr int CB = 32 / RJ;     // items merged per batch: 32 loads in flight per lane
+    for (int k = 0; k < n; ++k) {
+      const int slot = k % kPubSlots;
+      if (!warp_wait(&ms->pub_full[slot], (k / kPubSlots) & 1, ms, p.status)) break;
+      const ItemRef it = item_of(p, k);
+      // One partial per item: the two warpgroups' statistics combined here.
+      float2 *mine = p.partial + ((size_t)it.unit * p.n_ch + it.chunk) * C::R;
+#pragma unroll
+      for (int j = 0; j < RJ; ++j) {
+        const int r = lane + 32 * j;
+        float2 a = ms->pstat[slot][0][r];
+        const float2 b = ms->pstat[slot][1][r];
+        combine(a.x, a.y, b.x, b.y);
+        mine[r] = a;
+      }
+      __syncwarp();  // all lanes' rows are written (and the slot read) before lane 0 goes on
+      int last = 0;
+      if (lane == 0) {
+        mbar_arrive(&ms->pub_empty[slot]);
+        __threadfence();  // the item's partial becomes visible GPU-wide before it is counted
+        last = atomicAdd(&p.ctrl[it.unit], 1) == p.n_ch - 1;
+      }
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        // Last item of the unit: merge its n_ch partials per row.
+        __threadfence();
+        const float2 *part = p.partial + (size_t)it.unit * p.n_ch * C::R;
+        float mm[RJ], ll[RJ];
+#pragma unroll
+        for (int j = 0; j < RJ; ++j) {
+          mm[j] = -INFINITY;
+          ll[j] = 0.f;
+        }
+        for (int c0 = 0; c0 < p.n_ch; c0 += CB) {
+          float2 q[CB][RJ];
+#pragma unroll
+          for (int c = 0; c < CB; ++c)
+#pragma unroll
+            for (int j = 0; j < RJ; ++j)
+              q[c][j] = c0 + c < p.n_ch ? __ldcg(&part[(size_t)(c0 + c) * C::R + lane + 32 * j])
+                                        : make_float2(-INFINITY, 0.f);
+#pragma unroll
+          for (int c = 0; c < CB; ++c)
+#pragma unroll
+            for (int j = 0; j < RJ; ++j) combine(mm[j], ll[j], q[c][j].x, q[c][j].y);
+        }
+#pragma unroll
+        for (int j = 0; j < RJ; ++j)
+          p.lognorm[(size_t)it.unit * C::R + lane + 32 * j] = mm[j] + __log2f(ll[j]);
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release(&p.ctrl[p.units + it.unit], 1);
+      }
     }
   } else {
     // ------------------------------------------------ epilogue warpgroups
@@ -431,21 +498,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lrow = quarter * 32 + lane;      // row (pass 1) or key (pass 2) in the tile
     const int wtid = threadIdx.x - 64 - wg * 128;  // 0..127 within the warpgroup
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
-    int icount = 0, tcount = 0;
-    for (;;) {
-      const int slot = icount % kItemSlots;
-      if (!warp_wait(&ms->item_full[slot], (icount / kItemSlots) & 1, ms, p.status)) break;
-      const Item it = ms->items[slot];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ms->item_empty[slot]);
-      ++icount;
-      if (!it.pass) break;
-      int t0, t1;
-      item_tiles(p, it, t0, t1);
-      // Inside an item every warp follows the same control flow even if a wait
-      // gives up (the tile is then skipped), so that the named barriers below
-      // are always reached by all of their threads.
-      if (it.pass == 1) {
+    int tcount = 0;
+    // Inside an item every warp follows the same control flow even if a wait
+    // gives up (the tile is then skipped), so that the named barriers below
+    // are always reached by all of their threads.
+    for (int k = 0; k <= n; ++k) {
+      if (k < n) {
+        // ---------------- pass 1 of item k
+        const ItemRef it = item_of(p, k);
+        int t0, t1;
+        tiles_of(p, it, 1, t0, t1);
         float m[NR], l[NR];
         int last_vis[NR];
 #pragma unroll
@@ -472,94 +534,69 @@ __global__ void __launch_bounds__(kThreads, 1)
               __syncwarp();
               if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
             }
-            float tmax = -INFINITY;
-            if (!masked) {
-#pragma unroll
-              for (int c = 0; c < 4; ++c)
-#pragma unroll
-                for (int j = 0; j < 32; ++j) tmax = fmaxf(tmax, __uint_as_float(x[c][j]));
-            } else {
+            if (masked) {  // keys this row cannot see (causal window, past T) -> -inf
 #pragma unroll
               for (int c = 0; c < 4; ++c)
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
-                  if (t * kTile + c * 32 + j <= last_vis[nr])
-                    tmax = fmaxf(tmax, __uint_as_float(x[c][j]));
+                  if (t * kTile + c * 32 + j > last_vis[nr]) x[c][j] = 0xff800000u;
             }
+            // Eight independent chains keep the max and the sum off one long
+            // dependency chain.
+            float mx[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) mx[i] = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+              for (int j = 0; j < 32; ++j) mx[j & 7] = fmaxf(mx[j & 7], __uint_as_float(x[c][j]));
+            const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
             if (tmax == -INFINITY) continue;
             const float mnew = fmaxf(m[nr], tmax * p.scale2);
-            float s = 0.f;
-            if (!masked) {
+            float sv[8];
 #pragma unroll
-              for (int c = 0; c < 4; ++c)
+            for (int i = 0; i < 8; ++i) sv[i] = 0.f;
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  s += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
-            } else {
+            for (int c = 0; c < 4; ++c)
 #pragma unroll
-              for (int c = 0; c < 4; ++c)
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  if (t * kTile + c * 32 + j <= last_vis[nr])
-                    s += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
-            }
+              for (int j = 0; j < 32; ++j)
+                sv[j & 7] += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
+            const float s = ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
             l[nr] = l[nr] * fast_exp2(m[nr] - mnew) + s;
             m[nr] = mnew;
           }
         }
-        // Combine the two warpgroups' row stats; warpgroup 0 publishes them.
-        if (wg == 1) {
+        // This warpgroup's row statistics of the item go to the publisher warp
+        // through a shared-memory slot.
+        const int slot = k % kPubSlots;
+        warp_wait(&ms->pub_empty[slot], ((k / kPubSlots) & 1) ^ 1, ms, p.status);
 #pragma unroll
-          for (int nr = 0; nr < NR; ++nr) ms->xch[nr * 128 + lrow] = make_float2(m[nr], l[nr]);
+        for (int nr = 0; nr < NR; ++nr) ms->pstat[slot][wg][nr * 128 + lrow] = make_float2(m[nr], l[nr]);
+        __syncwarp();  // every lane's rows are written before lane 0 arrives
+        if (lane == 0) mbar_arrive(&ms->pub_full[slot]);
+      }
+      if (k >= 1) {
+        // ---------------- pass 2 of item k - 1
+        const ItemRef it = item_of(p, k - 1);
+        int t0, t1;
+        tiles_of(p, it, 2, t0, t1);
+        if (t1 > t0) {
+          if (wtid == 0) wait_ready(&p.ctrl[p.units + it.unit], ms, p.status);
+          named_bar_sync(3 + wg, 128);
+          for (int r = wtid; r < C::R; r += 128)
+            ms->off[wg][r] = __ldcg(&p.lognorm[(size_t)it.unit * C::R + r]);
+          named_bar_sync(3 + wg, 128);
         }
-        named_bar(1, 256);
-        if (wg == 0) {
-          const size_t prow = ((size_t)it.unit * p.n_ch1 + it.chunk) * C::R;
-#pragma unroll
-          for (int nr = 0; nr < NR; ++nr) {
-            const float2 o = ms->xch[nr * 128 + lrow];
-            combine(m[nr], l[nr], o.x, o.y);
-            p.partial[prow + nr * 128 + lrow] = make_float2(m[nr], l[nr]);
-          }
-          __threadfence();
-          named_bar(2, 128);
-          if (wtid == 0) {
-            const int done = atomicAdd(&p.ctrl[32 + it.unit], 1);
-            ms->last_flag = (done == p.n_ch1 - 1);
-          }
-          named_bar(2, 128);
-          if (ms->last_flag) {
-            __threadfence();
-#pragma unroll
-            for (int nr = 0; nr < NR; ++nr) {
-              const int r = nr * 128 + lrow;
-              float mm = -INFINITY, ll = 0.f;
-              for (int c = 0; c < p.n_ch1; ++c) {
-                const float2 q = __ldcg(&p.partial[((size_t)it.unit * p.n_ch1 + c) * C::R + r]);
-                combine(mm, ll, q.x, q.y);
-              }
-              p.lognorm[(size_t)it.unit * C::R + r] = mm + __log2f(ll);
-            }
-            __threadfence();
-            named_bar(2, 128);
-            if (wtid == 0) st_release(&p.ctrl[32 + p.units + it.unit], 1);
-          }
-        }
-        named_bar(1, 256);
-      } else {
-        // pass 2: wait for the unit's row statistics, then vote per key
-        if (wtid == 0) wait_ready(&p.ctrl[32 + p.units + it.unit], ms, p.status);
-        named_bar(3 + wg, 128);
-        for (int r = wtid; r < C::R; r += 128)
-          ms->off[wg][r] = __ldcg(&p.lognorm[(size_t)it.unit * C::R + r]);
-        named_bar(3 + wg, 128);
         const float4 *off4 = (const float4 *)ms->off[wg];
         for (int t = t0; t < t1; ++t, ++tcount) {
           if ((tcount & 1) != wg) continue;
           const int as = tcount % C::NA;
           if (!warp_wait(&ms->acc_full[as], (tcount / C::NA) & 1, ms, p.status)) continue;
           tc_fence_after();
-          float vote = 0.f;
+          float vs[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) vs[i] = 0.f;
           const uint32_t base = tmem + lane_addr + as * C::ACC_COLS;
 #pragma unroll
           for (int c4 = 0; c4 < NR; ++c4) {
@@ -577,12 +614,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int j = 0; j < 32; j += 4) {
                 const float4 o = off4[(c4 * 128 + c * 32 + j) >> 2];
-                vote += fast_exp2(fmaf(__uint_as_float(x[c][j + 0]), p.scale2, -o.x));
-                vote += fast_exp2(fmaf(__uint_as_float(x[c][j + 1]), p.scale2, -o.y));
-                vote += fast_exp2(fmaf(__uint_as_float(x[c][j + 2]), p.scale2, -o.z));
-                vote += fast_exp2(fmaf(__uint_as_float(x[c][j + 3]), p.scale2, -o.w));
+                const int h = (j >> 2) & 1;  // two chains per 4 columns: 8 in flight
+                vs[4 * h + 0] += fast_exp2(fmaf(__uint_as_float(x[c][j + 0]), p.scale2, -o.x));
+                vs[4 * h + 1] += fast_exp2(fmaf(__uint_as_float(x[c][j + 1]), p.scale2, -o.y));
+                vs[4 * h + 2] += fast_exp2(fmaf(__uint_as_float(x[c][j + 2]), p.scale2, -o.z));
+                vs[4 * h + 3] += fast_exp2(fmaf(__uint_as_float(x[c][j + 3]), p.scale2, -o.w));
               }
           }
+          const float vote = ((vs[0] + vs[1]) + (vs[2] + vs[3])) + ((vs[4] + vs[5]) + (vs[6] + vs[7]));
           const int key = t * kTile + lrow;
           if (key < p.P) p.votes[(size_t)it.unit * p.P + key] = vote;
         }
@@ -591,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   tc_fence_before();
-  __syncwarp();  // lanes 1..31 of the producer and MMA warps wait for lane 0 here
+  __syncwarp();  // idle lanes of the single-thread roles wait for their lane 0 here
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -663,33 +702,33 @@ cudaError_t launch_nr(const LayerGeom &g, const void *q_win, const void *k, cons
   p.G = g.G;
   p.n_tiles1 = (g.T + kTile - 1) / kTile;
   p.n_tiles2 = (g.P + kTile - 1) / kTile;
-  // tiles per item: enough items to keep every SM busy, at most 8
-  int chunk = (p.n_tiles1 * g.units) / (3 * sms);
-  p.chunk = chunk < 1 ? 1 : (chunk > 8 ? 8 : chunk);
-  p.n_ch1 = (p.n_tiles1 + p.chunk - 1) / p.chunk;
-  p.n_ch2 = (p.n_tiles2 + p.chunk - 1) / p.chunk;
-  // units per group: about 48 MB of keys, so that two groups stay in L2
-  const long long unit_bytes = (long long)g.T * 256;
-  int gu = (int)((48ll << 20) / unit_bytes);
-  p.group_units = gu < 1 ? 1 : (gu > g.units ? g.units : gu);
-  p.n_groups = (g.units + p.group_units - 1) / p.group_units;
-  p.n_items = g.units * (p.n_ch1 + p.n_ch2);
+  // Tiles per item: at least kMinTilesPerItem (hand-offs are per item), and
+  // enough that a unit has no more items than there are SMs (deadlock-free
+  // schedule, see the header comment).
+  const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
+  p.tpi = tpi_min > kMinTilesPerItem ? tpi_min : kMinTilesPerItem;
+  p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
+  p.total_items = g.units * p.n_ch;
   p.scale2 = g.scale2;
   p.partial = ws.row_partial;
   p.lognorm = ws.row_lognorm;
   p.votes = votes;
   p.ctrl = ws.counters;
   p.status = status;
-  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * (32 + 2 * g.units), st);
+  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * g.units, st);
   if (e != cudaSuccess) return e;
   constexpr int smem = smem_bytes<NR>();
   static_assert(smem <= 227 * 1024, "shared memory budget");
   e = cudaFuncSetAttribute(score_tc_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const int grid = p.n_items < sms ? p.n_items : sms;
-  score_tc_kernel<NR><<<grid, kThreads, smem, st>>>(kmap, qmap, p);
+  const int grid = p.total_items < sms ? p.total_items : sms;
+  // Cooperative launch: every CTA resident at once, which the cross-CTA waits
+  // of the schedule rely on.
+  void *args[] = {(void *)&kmap, (void *)&qmap, (void *)&p};
+  e = cudaLaunchCooperativeKernel((const void *)score_tc_kernel<NR>, dim3(grid), dim3(kThreads),
+                                  args, (size_t)smem, st);
   count_launches(1);
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace

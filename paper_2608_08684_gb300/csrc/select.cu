@@ -22,26 +22,14 @@ namespace {
 constexpr int kThreads = kSelectThreads;
 constexpr int kWarps = kThreads / 32;
 constexpr int kBins = 2048;
+// Shared words after the histogram: scan scratch [0, 33), control [40, 48),
+// per-warp exclusive counts [0, 32) and [48, 80) during the compaction.
+constexpr int kCtrlWords = 128;
 
 // Order-preserving map float -> uint32 (larger float, larger key); -0 folds to +0.
 __device__ __forceinline__ uint32_t order_key(float x) {
   const uint32_t b = __float_as_uint(x + 0.0f);
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-}
-
-__device__ __forceinline__ float pooled_score(const float *v, int P, int t, int half, int type) {
-  const int lo = max(0, t - half), hi = min(P - 1, t + half);
-  if (type == RIPPLE_POOL_MAX) {
-    float m = v[lo];
-    for (int j = lo + 1; j <= hi; ++j) m = fmaxf(m, v[j]);
-    return m;
-  }
-  if (type == RIPPLE_POOL_AVG) {
-    float s = 0.f;
-    for (int j = lo; j <= hi; ++j) s = __fadd_rn(s, v[j]);
-    return __fdiv_rn(s, (float)(hi - lo + 1));
-  }
-  return v[t];
 }
 
 // Exclusive block-wide prefix sum of one int per thread; *total gets the sum.
@@ -80,7 +68,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
   uint32_t *hist = sm;                              // [kBins]
   int *warp_tot = (int *)(sm + kBins);              // [33]
   int *ctrl = warp_tot + 40;                        // [8] control words
-  uint32_t *keys = in_smem ? sm + kBins + 48 : keys_global + (size_t)blockIdx.x * g.P;
+  uint32_t *keys = in_smem ? sm + kBins + kCtrlWords : keys_global + (size_t)blockIdx.x * g.P;
 
   const int unit = blockIdx.x;
   const int P = g.P, K = n_keep - g.W;
@@ -95,8 +83,42 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
     return;
   }
 
+  // Pooling: each warp step loads 32 consecutive votes (coalesced) and the
+  // lanes away from the edges take their window through shuffles.
   const int half = g.pool_kernel / 2;
-  for (int t = tid; t < P; t += kThreads) keys[t] = order_key(pooled_score(v, P, t, half, g.pool_type));
+  const int lane = tid & 31, wid = tid >> 5;
+  const int step = 32 - 2 * half;
+  for (int seg = wid * step; seg < P; seg += kWarps * step) {
+    const int src = seg - half + lane;
+    const bool in = src >= 0 && src < P;
+    const float x = in ? v[src] : 0.f;
+    float r;
+    if (g.pool_type == RIPPLE_POOL_MAX) {
+      r = in ? x : -INFINITY;
+      const float own = r;
+      for (int d = 1; d <= half; ++d) {
+        r = fmaxf(r, __shfl_up_sync(0xffffffffu, own, d));
+        r = fmaxf(r, __shfl_down_sync(0xffffffffu, own, d));
+      }
+    } else if (g.pool_type == RIPPLE_POOL_AVG) {
+      // ascending positions from zero, like the definition's sum
+      float s = 0.f;
+      int cnt = 0;
+      for (int d = -half; d <= half; ++d) {
+        const float xv = d < 0 ? __shfl_up_sync(0xffffffffu, x, -d)
+                               : __shfl_down_sync(0xffffffffu, x, d);
+        const int pos = src + d;
+        if (pos >= 0 && pos < P) {
+          s = __fadd_rn(s, d == 0 ? x : xv);
+          ++cnt;
+        }
+      }
+      r = __fdiv_rn(s, (float)cnt);
+    } else {
+      r = x;
+    }
+    if (lane >= half && lane < 32 - half && src < P) keys[src] = order_key(r);
+  }
   __syncthreads();
 
   // Radix select of the K-th largest key.
@@ -142,23 +164,50 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
   const int take_eq = remaining;  // keys equal to tau that are kept (>= 1)
 
   // Ordered compaction: all keys > tau, plus the first take_eq keys == tau.
-  int carry_gt = 0, carry_eq = 0;
-  for (int base = 0; base < P; base += kThreads) {
-    const int t = base + tid;
-    int gt = 0, eq = 0;
-    if (t < P) {
-      const uint32_t u = keys[t];
-      gt = u > tau;
-      eq = u == tau;
+  // Each warp owns one contiguous index range: it counts, one block scan gives
+  // every warp its output offsets, then it writes its range in order.
+  const int per = ((P + kWarps - 1) / kWarps + 31) & ~31;
+  const int r0 = min(P, wid * per), r1 = min(P, r0 + per);
+  int cgt = 0, ceq = 0;
+  for (int b = r0; b < r1; b += 32) {
+    const int t = b + lane;
+    const uint32_t u = t < r1 ? keys[t] : 0u;
+    cgt += __popc(__ballot_sync(0xffffffffu, t < r1 && u > tau));
+    ceq += __popc(__ballot_sync(0xffffffffu, t < r1 && u == tau));
+  }
+  int *wgt = warp_tot, *weq = warp_tot + 40 + 8;  // [32] each
+  if (lane == 0) {
+    wgt[wid] = cgt;
+    weq[wid] = ceq;
+  }
+  __syncthreads();
+  if (wid == 0) {
+    int a = wgt[lane], e = weq[lane];
+    int ia = a, ie = e;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int ya = __shfl_up_sync(0xffffffffu, ia, o), ye = __shfl_up_sync(0xffffffffu, ie, o);
+      if (lane >= o) {
+        ia += ya;
+        ie += ye;
+      }
     }
-    int total;
-    const int before = block_exclusive_scan(gt | (eq << 16), warp_tot, &total);
-    const int gt_before = before & 0xffff, eq_before = before >> 16;
-    const int eq_rank = carry_eq + eq_before;
-    if (gt || (eq && eq_rank < take_eq)) out[carry_gt + gt_before + min(eq_rank, take_eq)] = t;
-    carry_gt += total & 0xffff;
-    carry_eq += total >> 16;
-    if (carry_gt + min(carry_eq, take_eq) >= K) break;
+    wgt[lane] = ia - a;
+    weq[lane] = ie - e;
+  }
+  __syncthreads();
+  int gt_before = wgt[wid], eq_before = weq[wid];
+  const uint32_t below = (1u << lane) - 1u;
+  for (int b = r0; b < r1; b += 32) {
+    const int t = b + lane;
+    const uint32_t u = t < r1 ? keys[t] : 0u;
+    const bool gt = t < r1 && u > tau, eq = t < r1 && u == tau;
+    const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
+    const int g_rank = gt_before + __popc(bg & below);
+    const int e_rank = eq_before + __popc(be & below);
+    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = t;
+    gt_before += __popc(bg);
+    eq_before += __popc(be);
   }
 }
 
@@ -167,7 +216,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
 cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
                           int n_keep, int32_t *idx, cudaStream_t st) {
   const int in_smem = g.P <= kSelectSmemKeys;
-  const size_t smem = sizeof(uint32_t) * (kBins + 48 + (in_smem ? g.P : 0));
+  const size_t smem = sizeof(uint32_t) * (kBins + kCtrlWords + (in_smem ? g.P : 0));
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
