@@ -136,6 +136,32 @@ def run_case(args):
                       "peak_source": src}), flush=True)
 
 
+def profile_traffic(profile, sources, alg_bytes):
+    """DRAM traffic (read + write bytes) of one launch from a committed ncu
+    summary under profiles/, scaled from the captured launch to this one by
+    algorithmic bytes. None when the kernel's sources changed since the
+    capture (their hash differs) or the summary is missing."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", profile)
+    try:
+        fields = {}
+        for line in open(path):
+            if ":" in line and not line.startswith(("|", "#", " ")):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+        h = hashlib.sha256()
+        for s in sources:
+            with open(os.path.join(ROOT, "paper_2608_08684_gb300", "csrc", s), "rb") as f:
+                h.update(f.read())
+        if h.hexdigest()[:16] != fields["source_sha256"]:
+            return None
+        traffic = float(fields["traffic_bytes_per_launch"])
+        captured = float(fields["algorithmic_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+    return round(traffic * alg_bytes / captured)
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -306,6 +332,30 @@ def elapsed_ms(pairs):
     return [a.elapsed_time(b) for a, b in pairs]
 
 
+def replica_workload(wl, rank):
+    """Rank r of a multi-GPU run serves its own independent batch (replicas:
+    the path has no exchange step), seeded apart from the other ranks."""
+    return wl.replace(seed=wl.seed + 1000 * rank) if rank else wl
+
+
+def max_over_ranks(ms, world, device):
+    """The timed region's length as the slowest rank saw it."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    tt = torch.tensor([ms], device=device, dtype=torch.float64)
+    dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+    return float(tt.item())
+
+
+def job_throughput(total_ms, steps, tokens_per_rank, world):
+    """(ms per step, whole-job tokens/s): every rank processed its own batch
+    within the max-over-ranks time."""
+    ms_per_step = total_ms / steps
+    return ms_per_step, tokens_per_rank * world / (ms_per_step / 1e3)
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     import torch.distributed as dist
@@ -325,7 +375,7 @@ def run_ours(args, rank, world, local_rank):
 
     wl = synth.WORKLOADS[args.workload]
     # independent replicas: every rank serves its own batch (weak scaling)
-    wl = wl.replace(seed=wl.seed + 1000 * rank) if rank else wl
+    wl = replica_workload(wl, rank)
     st = Serving(R, synth, wl, device)
     torch.cuda.synchronize()
 
@@ -353,14 +403,9 @@ def run_ours(args, rank, world, local_rank):
         barrier()
     launches = R.ripple_kernel_launches() - launches0
     assert int(st.status.item()) == 0
-    total_ms = t0.elapsed_time(t1)
-    if world > 1:
-        tt = torch.tensor([total_ms], device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
-    ms_per_step = total_ms / args.steps
+    total_ms = max_over_ranks(t0.elapsed_time(t1), world, device)
+    ms_per_step, value = job_throughput(total_ms, args.steps, wl.batch * wl.seq_len, world)
     tokens = wl.batch * wl.seq_len * world
-    value = tokens / (ms_per_step / 1e3)
 
     comp_ms = elapsed_ms(timers[0])
     dec_ms = elapsed_ms(timers[1])
@@ -371,14 +416,20 @@ def run_ours(args, rank, world, local_rank):
     dec_gbs = st.decode_bytes_per_step() / (dec_avg / 1e3) / 1e9
     comp_total = comp_avg
     dec_total = dec_avg * wl.decode_steps
+    dec_traffic = profile_traffic("decode_kernel_llama3-8b_B4_T32768.md",
+                                  ["decode.cu", "common.cuh"], st.decode_bytes_per_step()) \
+        if wl.name.startswith("llama3-8b-32L-32q8kv-d128-B4-T32768") else None
     roof_dec = {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(dec_gbs / hbm, 4), "traffic": None,
-                "kernel": "ripple_decode_attn (decode_partial + decode_combine)",
+                "frac": round(dec_gbs / hbm, 4), "traffic": dec_traffic,
+                "traffic_source": ("ncu dram bytes of the first decode step "
+                                   "(profiles/decode_kernel_llama3-8b_B4_T32768.md), scaled "
+                                   "by algorithmic bytes") if dec_traffic else None,
+                "kernel": "decode_kernel (ripple_decode_attn, one launch per step)",
                 "bytes_per_launch": round(st.decode_bytes_per_step()),
                 "ms_per_launch": round(dec_avg, 5), "peak_source": hbm_src}
     roof_comp = {"bound": "hbm", "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s",
                  "frac": round(comp_gbs / hbm, 4), "traffic": None,
-                 "kernel": "ripple_compress_layer x all layers",
+                 "kernel": "score_tc_kernel + select_kernel + gather_kernel (ripple_compress_layer, all layers)",
                  "bytes_per_launch": round(st.compress_bytes()),
                  "ms_per_launch": round(comp_avg, 4), "peak_source": hbm_src}
     dominant = roof_dec if dec_total >= comp_total else roof_comp
@@ -474,26 +525,29 @@ def measure_e2e(st, args, torch, tokens):
 # ----------------------------------------------------------------- CPU oracle
 
 
-def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s):
+def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s, layers=None):
     """Times the oracle on a bounded sample of compression units and decode
-    groups and extrapolates to one full step. Returns (step seconds, sample text)."""
+    groups and extrapolates to one full step. Returns (step seconds, sample text).
+    `layers` limits the compression sample to those layers (all by default)."""
     import numpy as np
 
     from oracle import ripple_oracle as O
     scale = 1.0 / math.sqrt(wl.head_dim)
     units_total = wl.n_layers * wl.batch * wl.n_kv_heads
-    # compression sample: units of the largest-budget layer, round robin over (b, h)
-    layer = int(np.argmax(budgets))
+    # compression sample: units round robin over the sampled layers (each
+    # layer's own budget), then over (b, h), until about 3/4 of the time target
+    layers = list(range(wl.n_layers)) if layers is None else list(layers)
     t_comp, n_comp = 0.0, 0
-    while t_comp < 0.75 * target_s and n_comp < wl.batch * wl.n_kv_heads:
-        b, h = divmod(n_comp, wl.n_kv_heads)
+    while t_comp < 0.75 * target_s and n_comp < len(layers) * wl.batch * wl.n_kv_heads:
+        layer = layers[n_comp % len(layers)]
+        b, h = divmod((n_comp // len(layers)) % (wl.batch * wl.n_kv_heads), wl.n_kv_heads)
         q, k, v = get_unit(layer, b, h)
         t = time.perf_counter()
         O.compress_unit(q, k, v, budgets[layer], wl.window, scale, wl.pool_kernel)
         t_comp += time.perf_counter() - t
         n_comp += 1
-    # decode sample: one (layer, b, h) group per layer, over min(8, steps) steps
-    steps = min(8, wl.decode_steps)
+    # decode sample: one (layer, b, h) group per layer, over the first steps
+    steps = min(16, wl.decode_steps)
     t_dec, n_dec = 0.0, 0
     for layer in range(wl.n_layers):
         if t_dec > 0.25 * target_s:
@@ -511,7 +565,8 @@ def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s):
     per_group_step = t_dec / n_dec
     step_s = per_unit * units_total + per_group_step * (
         wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps)
-    sample = (f"{n_comp} compression units of layer {layer} (T={wl.seq_len}) and {n_dec} "
+    sample = (f"{n_comp} compression units (T={wl.seq_len}, round robin over {len(layers)} "
+              f"layers) and {n_dec} "
               f"decode (group, step) pairs; extrapolated to {units_total} units and "
               f"{wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps} group-steps")
     return step_s, sample, t_comp + t_dec
@@ -578,11 +633,15 @@ def run_reference(args, rank, world):
     budgets = O.alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
                               wl.global_budget)
     n_keep = [O.keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    # Four sampled layers (largest and smallest budget, two in between), each
+    # generated once on the host.
+    by_budget = sorted(range(wl.n_layers), key=lambda i: budgets[i])
+    sample_layers = sorted({by_budget[-1], by_budget[0], by_budget[len(by_budget) // 3],
+                            by_budget[2 * len(by_budget) // 3]})
     layer_cache = {}
 
     def layer_tensors(layer):
         if layer not in layer_cache:
-            layer_cache.clear()
             layer_cache[layer] = (synth.layer_window_queries(wl, layer),
                                   synth.layer_keys(wl, layer), synth.layer_values(wl, layer))
         return layer_cache[layer]
@@ -596,7 +655,8 @@ def run_reference(args, rank, world):
     per_step = max(2.0, min(args.cpu_seconds, 120.0 / max(1, args.steps + args.warmup)))
     times, sample = [], ""
     for i in range(args.warmup + args.steps):
-        step_s, sample, _ = oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, per_step)
+        step_s, sample, _ = oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, per_step,
+                                               layers=sample_layers)
         if i >= args.warmup:
             times.append(step_s)
     step_s = statistics.mean(times)
