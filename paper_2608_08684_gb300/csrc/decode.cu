@@ -26,6 +26,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "decode.cuh"
 #include "kernels.cuh"
 
 namespace ripple {
@@ -60,22 +61,6 @@ struct DecCfg {
   static_assert(NIT >= 1 && RPW % RPI == 0, "rows per warp");
   static_assert(PPL * S == PIECES && HL >= 1, "lanes per row");
   static_assert(DL % 2 == 0 && DV % 2 == 0, "fp32x2 pairs");
-};
-
-struct DecParams {
-  int L, B, Hq, Hkv, G;
-  float scale2;
-  const void *q, *k_new, *v_new;
-  int32_t *lens;
-  float *out;
-  float *ws_o;      // [items][G][D] unnormalised partial outputs
-  float2 *ws_ml;    // [items][G] (max, sum) of each partial
-  int *ctrl;        // [0] item counter, [1] exit counter, [2 + group] items done
-  int32_t *status;
-  const void *kc[RIPPLE_MAX_LAYERS];
-  const void *vc[RIPPLE_MAX_LAYERS];
-  int cap[RIPPLE_MAX_LAYERS];
-  int order[RIPPLE_MAX_LAYERS];  // layers by decreasing capacity
 };
 
 template <typename Tin, int D, int G>
@@ -660,7 +645,9 @@ ripple_status run(const ripple_decode_desc *desc, const DecParams &p, void *stre
   cudaStream_t st = (cudaStream_t)stream;
   if (cudaMemsetAsync(p.ctrl, 0, ctrl_bytes(desc), st) != cudaSuccess) return RIPPLE_ECUDA;
   cudaError_t e;
-  if (desc->dtype == RIPPLE_F32)
+  if (decode_tc_supported(desc, item_rows(desc)))
+    e = launch_decode_tc(p, st);
+  else if (desc->dtype == RIPPLE_F32)
     e = desc->head_dim == 64 ? launch_d<float, 64>(p, st) : launch_d<float, 128>(p, st);
   else
     e = desc->head_dim == 64 ? launch_d<__nv_bfloat16, 64>(p, st)

@@ -66,6 +66,14 @@ DECODE_SHAPES = [
                           dtype="bf16", seed=42), [127, 513]),
     ("bf16-d64-G1", dict(n_layers=2, batch=2, n_q_heads=3, n_kv_heads=3, head_dim=64,
                          dtype="bf16", seed=43), [64, 200]),
+    # groups split over several 2048-row work items, item edges and a ragged tail
+    ("bf16-d128-G4-split", dict(n_layers=4, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
+                                dtype="bf16", kv_dist="scaled_sinks", seed=47),
+     [2047, 2048, 2049, 4500]),
+    ("bf16-d128-G1", dict(n_layers=2, batch=2, n_q_heads=2, n_kv_heads=2, head_dim=128,
+                          dtype="bf16", seed=48), [0, 129]),
+    ("bf16-d128-G2", dict(n_layers=2, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=128,
+                          dtype="bf16", kv_dist="scaled_sinks", seed=49), [31, 4095]),
 ]
 
 
@@ -116,6 +124,27 @@ def test_decode_full_cache_reports_and_skips(lib):
     assert int(s.status.item()) == lib.EFULL
     assert s.lens.cpu().tolist() == [10, 5]
     assert np.all(got[0] == 0.0) and np.any(got[1] != 0.0)
+    assert torch.equal(s.k[0].cpu(), kc[0])
+
+
+def test_decode_full_cache_bf16_d128(lib):
+    # the tensor-core path (bf16, d = 128): a full layer is skipped and reported
+    wl = synth.WORKLOADS["tiny"].replace(n_layers=2, dtype="bf16", head_dim=128, n_q_heads=8,
+                                         n_kv_heads=2, seed=50)
+    caps = [300, 300]
+    kc, vc = zip(*[synth.decode_caches(wl, i, 300) for i in range(2)])
+    s = Session(lib, wl, range(2), caps, [300, 200], kc, vc)
+    q, kn, vn = synth.decode_inputs(wl, 0)
+    got = s.step(q, kn, vn)
+    assert int(s.status.item()) == lib.EFULL
+    assert s.lens.cpu().tolist() == [300, 201]
+    assert np.all(got[0] == 0.0)
+    rows_k = [[[synth.to_f64(kc[1][b, h, :200]) for h in range(wl.n_kv_heads)]
+               for b in range(wl.batch)]]
+    rows_v = [[[synth.to_f64(vc[1][b, h, :200]) for h in range(wl.n_kv_heads)]
+               for b in range(wl.batch)]]
+    ref = _oracle_step(wl, rows_k, rows_v, q[1:], kn[1:], vn[1:])
+    assert np.abs(got[1:] - ref).max() <= C.DECODE_ATOL
     assert torch.equal(s.k[0].cpu(), kc[0])
 
 
