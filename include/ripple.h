@@ -218,7 +218,18 @@ ripple_status ripple_decode_workspace_bytes(const ripple_decode_desc *desc,
  * lens         device int32 [L]: rows in use per layer (same for every b, h);
  *              read, then incremented by one per layer
  * out          device fp32 [L][B][Hq][d]
- * workspace    device scratch of at least ripple_decode_workspace_bytes bytes
+ * workspace    device scratch of at least ripple_decode_workspace_bytes bytes.
+ *              Its leading block holds the step's work counters. For bf16,
+ *              d = 128 and at most 80 layers (the tensor-core path) every call
+ *              leaves that block at zero, and the library clears it only when
+ *              the workspace differs from the one its previous such call on
+ *              the device used; so between consecutive calls with the same
+ *              workspace the caller must not write into it (another buffer
+ *              is fine). After a call that ended with RIPPLE_ETIMEOUT in
+ *              *dev_status, pass a different workspace or zero the block.
+ * Consecutive calls on one stream may overlap: a call's thread blocks may
+ * start while the previous call's last blocks finish; they read nothing the
+ * previous call writes before it has completed.
  * A layer with lens[l] >= caps_host[l] (or lens[l] < 0) is not appended to,
  * its output rows are zero, its length is unchanged, and RIPPLE_EFULL is
  * written to *dev_status.
@@ -253,9 +264,13 @@ ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
  * - Returns RIPPLE_EWORKSPACE, before enqueuing anything, when the step needs
  *   more scratch than the array holds (ripple_decode_workspace_bytes(desc,
  *   caps) > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
- * - Every call on a device shares the one array. Each call clears the
- *   counters it uses at its start (a memset enqueued on `stream`) and rewrites
- *   every partial it reads, so nothing carries over from the previous call.
+ * - Every call on a device shares the one array. Its counters start at zero
+ *   (the array is zero-initialised when the library is loaded) and every call
+ *   leaves them at zero (the tensor-core path resets them as it exits; other
+ *   paths clear them with a memset enqueued on `stream` first); every partial
+ *   a call reads it has rewritten, so nothing carries over from the previous
+ *   call. A call that ended with RIPPLE_ETIMEOUT may leave the counters
+ *   dirty: later calls of this entry point on that device are then invalid.
  *   Calls that may overlap on the GPU (different streams without ordering)
  *   race on it; order them, e.g. by issuing them on one stream.
  */

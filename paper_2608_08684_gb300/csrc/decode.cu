@@ -550,7 +550,9 @@ cudaError_t launch_d(const DecParams &p, cudaStream_t st) {
   }
 }
 
+// Cache rows per work item of the kernel that serves this descriptor.
 int item_rows(const ripple_decode_desc *d) {
+  if (decode_tc_supported(d)) return kTcItemRows;
   const int row_bytes = d->head_dim * (d->dtype == RIPPLE_F32 ? 4 : 2);
   return (kStageBytes / row_bytes) * kItemSub;
 }
@@ -643,11 +645,12 @@ ripple_status prepare(const ripple_decode_desc *desc, const void *q, const void 
 
 ripple_status run(const ripple_decode_desc *desc, const DecParams &p, void *stream) {
   cudaStream_t st = (cudaStream_t)stream;
+  if (decode_tc_supported(desc))
+    return launch_decode_tc(p, ctrl_bytes(desc), st) == cudaSuccess ? RIPPLE_OK : RIPPLE_ECUDA;
+  decode_tc_forget_ctrl(p.ctrl);
   if (cudaMemsetAsync(p.ctrl, 0, ctrl_bytes(desc), st) != cudaSuccess) return RIPPLE_ECUDA;
   cudaError_t e;
-  if (decode_tc_supported(desc, item_rows(desc)))
-    e = launch_decode_tc(p, st);
-  else if (desc->dtype == RIPPLE_F32)
+  if (desc->dtype == RIPPLE_F32)
     e = desc->head_dim == 64 ? launch_d<float, 64>(p, st) : launch_d<float, 128>(p, st);
   else
     e = desc->head_dim == 64 ? launch_d<__nv_bfloat16, 64>(p, st)
@@ -694,10 +697,12 @@ extern "C" ripple_status ripple_decode_attn(const ripple_decode_desc *desc, cons
 // have no way to hand this library a scratch buffer. For those callers the
 // step's control counters and split-K partials live in the file-scope device
 // array below instead of a caller workspace. Every GPU that loads the library
-// keeps it until the process exits; all calls on a device share it. Each call
-// clears the counters it needs at its start (a memset on the stream) and
-// fully rewrites the partials it reads, so no state carries over from the
-// previous call; calls that overlap on the GPU race on it.
+// keeps it until the process exits; all calls on a device share it. Its
+// counters start at zero (zero-initialised at load) and every call leaves them
+// at zero (the tensor-core kernel resets them as it exits, the other kernels
+// are preceded by a memset on the stream); every partial a call reads it has
+// rewritten, so no state carries over from the previous call. Calls that
+// overlap on the GPU race on it.
 
 static __device__ __align__(256) float
     g_decode_scratch[RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES / sizeof(float)];

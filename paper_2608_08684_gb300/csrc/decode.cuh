@@ -27,8 +27,13 @@ struct DecParams {
 
 // Tensor-core decode (bf16, d = 128, up to kTcMaxLayers layers per call).
 constexpr int kTcMaxLayers = 80;
-constexpr int kTcItemRows = 2048;  // cache rows per work item (16 tiles of 128)
-bool decode_tc_supported(const ripple_decode_desc *d, int item_rows);
-cudaError_t launch_decode_tc(const DecParams &p, cudaStream_t st);
+constexpr int kTcItemRows = 4096;  // cache rows per work item (32 tiles of 128)
+bool decode_tc_supported(const ripple_decode_desc *d);
+// Clears the counter block itself unless the previous tensor-core call on
+// this device left this block at zero.
+cudaError_t launch_decode_tc(const DecParams &p, size_t ctrl_bytes, cudaStream_t st);
+// The counter block at `ctrl` is no longer known to be zero (another kernel
+// used it).
+void decode_tc_forget_ctrl(const void *ctrl);
 
 }  // namespace ripple

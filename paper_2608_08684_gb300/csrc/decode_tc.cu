@@ -22,9 +22,9 @@
 // An item covering its whole group writes the output; otherwise it stores its
 // unnormalised partial and the group's last item combines them in item order.
 //
-// Warp roles (192 threads): warp 0 = producer (work items, queries, tile
-// loads), warp 1 = MMA issuer and TMEM owner, warps 2-5 = epilogue (TMEM lane
-// quarter = warp % 4). Every wait is bounded; on timeout the CTA raises
+// Warp roles (224 threads): warp 0 = tile producer (work items, key / value
+// tiles), warp 1 = MMA issuer and TMEM owner, warps 2-5 = epilogue (TMEM lane
+// quarter = warp % 4), warp 6 = per-item set-up (queries, new token). Every wait is bounded; on timeout the CTA raises
 // RIPPLE_ETIMEOUT, every role leaves its loop and TMEM is released.
 #include <math.h>
 
@@ -45,7 +45,7 @@ constexpr int kRing = 6;                    // K / V tile slots
 constexpr int kNS = 4;                      // score accumulators (16 TMEM columns each)
 constexpr int kStatSlots = 3;
 constexpr int kItemSlots = 4;
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
 constexpr int kOpBytes = 4096;              // a 16 x 128 bf16 operand (queries or P)
 constexpr uint32_t kSCol = 0;               // TMEM: scores  [kNS][16]
 constexpr uint32_t kOCol = 64;              //       outputs [2][4 warps][16]
@@ -62,7 +62,7 @@ struct Misc {
   uint64_t q_full[2], q_empty[2];
   uint64_t s_full[kNS], s_empty[kNS];
   uint64_t p_full[2], o_full[2], o_empty[2];
-  uint64_t item_full[kItemSlots], item_empty[kItemSlots];
+  uint64_t item_full[kItemSlots], item_empty[kItemSlots], new_full[kItemSlots];
   uint64_t mma_done;
   int item_id[kItemSlots];
   float s_new[kItemSlots][8];          // new token's scaled scores per head
@@ -155,6 +155,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int units = p.B * p.Hkv;
 
+  // Launched as a programmatic dependent of the previous step: let the next
+  // step's CTAs take SMs as this grid's CTAs leave, and wait here until the
+  // previous grid has finished and its writes (lengths, appended rows,
+  // counters) are visible.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   // Work list of this step from the current lengths (read once, before any
   // CTA can advance them: that happens after every CTA has exited).
   if (tid < p.L) {
@@ -186,7 +192,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kItemSlots; ++i) {
       mbar_init(&ms->item_full[i], 1);
-      mbar_init(&ms->item_empty[i], 5);  // MMA warp + 4 epilogue warps
+      mbar_init(&ms->item_empty[i], 6);  // MMA, set-up and 4 epilogue warps
+      mbar_init(&ms->new_full[i], 1);
     }
     mbar_init(&ms->mma_done, 1);
     ms->abort_flag = 0;
@@ -213,27 +220,66 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = ms->tmem_base;
 
   if (warp == 0) {
-    // ------------------------------------------------ producer warp
-    int icount = 0, lcount = 0, qcount = 0;  // items, tile loads, query operands
-    for (;; ++icount) {
-      const int slot = icount % kItemSlots;
-      int it = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
-      it = __shfl_sync(0xffffffffu, it, 0);
-      if (!warp_wait(&ms->item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, ms, p.status)) break;
-      if (it >= total) {
-        if (lane == 0) {
-          ms->item_id[slot] = total;
-          mbar_arrive(&ms->item_full[slot]);
+    // ------------------------------------------------ tile producer (one lane)
+    // Work items are fetched one ahead; an item is published to the other
+    // roles and its key / value tiles are issued at once, so the ring keeps
+    // streaming across item boundaries.
+    if (lane == 0) {
+      int lcount = 0;
+      int it = atomicAdd(&p.ctrl[0], 1);
+      for (int icount = 0;; ++icount) {
+        const int slot = icount % kItemSlots;
+        const int nxt = it < total ? atomicAdd(&p.ctrl[0], 1) : total;
+        if (!wait_bar(&ms->item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, ms, p.status)) break;
+        ms->item_id[slot] = min(it, total);
+        mbar_arrive(&ms->item_full[slot]);
+        if (it >= total) break;
+        const Item f = item_of(p, ms, it);
+        bool ok = true;
+        if (f.tiles > 0) {
+          const CUtensorMap *km = &tp.kmap[f.pos];
+          const CUtensorMap *vm = &tp.vmap[f.pos];
+          const int unit = f.b * p.Hkv + f.h;
+          const uint64_t pol = policy_evict_first();  // every cache row is read once
+          for (int j = 0; j < f.tiles && ok; ++j) {
+            const int y = f.r0 + j * kTile;
+            for (int kv = 0; kv < 2; ++kv, ++lcount) {
+              const int rs = lcount % kRing;
+              if (!wait_bar(&ms->kv_empty[rs], ((lcount / kRing) & 1) ^ 1, ms, p.status)) {
+                ok = false;
+                break;
+              }
+              mbar_arrive_expect_tx(&ms->kv_full[rs], kTileBytes);
+              uint8_t *dst = ring + rs * kTileBytes;
+              const CUtensorMap *m = kv ? vm : km;
+              tma_load_3d(dst, m, 0, y, unit, &ms->kv_full[rs], pol);
+              tma_load_3d(dst + kHalf, m, 64, y, unit, &ms->kv_full[rs], pol);
+            }
+          }
         }
-        break;
+        if (!ok) break;
+        it = nxt;
       }
+      // Let issued copies land before the CTA can exit (after an abort).
+      for (int j = max(0, lcount - kRing); j < lcount; ++j)
+        mbar_wait(&ms->kv_full[j % kRing], (j / kRing) & 1, nullptr, kWaitCycles / 4);
+    }
+  } else if (warp == 6) {
+    // ------------------------------------------------ per-item set-up warp
+    // Stages each item's queries as the score product's operand, and for a
+    // group's last item scores the new token and appends it to the cache.
+    int qcount = 0;
+    for (int icount = 0;; ++icount) {
+      const int slot = icount % kItemSlots;
+      if (!warp_wait(&ms->item_full[slot], (icount / kItemSlots) & 1, ms, p.status)) break;
+      const int it = ms->item_id[slot];
+      if (it >= total) break;
       const Item f = item_of(p, ms, it);
-      bool ok = true;
       if (!f.full) {
-        const int qs = qcount & 1;
         const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
         if (f.tiles > 0) {
-          ok = warp_wait(&ms->q_empty[qs], ((qcount >> 1) & 1) ^ 1, ms, p.status);
+          const int qs = qcount & 1;
+          const bool ok = warp_wait(&ms->q_empty[qs], ((qcount >> 1) & 1) ^ 1, ms, p.status);
           ++qcount;
           if (ok) {
             // the group's G query rows into the operand (16-byte pieces)
@@ -252,15 +298,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (f.chunk == f.nch - 1) {
           // The new token: its scores, and its append to the cache.
           const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * 256;
-          const __nv_bfloat16 *kn = (const __nv_bfloat16 *)((const uint8_t *)p.k_new + nb);
-          const __nv_bfloat16 *qn = (const __nv_bfloat16 *)p.q + qrow * 128;
+          const uint2 kn = reinterpret_cast<const uint2 *>((const uint8_t *)p.k_new + nb)[lane];
+          const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kn.x));
+          const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kn.y));
 #pragma unroll
           for (int g = 0; g < G; ++g) {
-            float s = 0.f;
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-              s = fmaf(__bfloat162float(qn[g * 128 + lane * 4 + e]),
-                       __bfloat162float(kn[lane * 4 + e]), s);
+            const uint2 qv =
+                reinterpret_cast<const uint2 *>((const uint8_t *)p.q + (qrow + g) * 256)[lane];
+            const float2 q01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&qv.x));
+            const float2 q23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&qv.y));
+            float s = fmaf(q01.x, k01.x, fmaf(q01.y, k01.y, fmaf(q23.x, k23.x, q23.y * k23.y)));
             s = warp_sum(s);
             if (lane == 0) ms->s_new[slot][g] = s * p.scale2;
           }
@@ -274,38 +321,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       __syncwarp();
       if (lane == 0) {
-        ms->item_id[slot] = it;
-        mbar_arrive(&ms->item_full[slot]);
+        mbar_arrive(&ms->new_full[slot]);
+        mbar_arrive(&ms->item_empty[slot]);
       }
-      if (!ok) break;
-      // Key and value tiles of the item, in ring order K0 V0 K1 V1 ...
-      if (lane == 0 && f.tiles > 0) {
-        const CUtensorMap *km = &tp.kmap[f.pos];
-        const CUtensorMap *vm = &tp.vmap[f.pos];
-        const int unit = f.b * p.Hkv + f.h;
-        for (int j = 0; j < f.tiles && ok; ++j) {
-          const int y = f.r0 + j * kTile;
-          for (int kv = 0; kv < 2; ++kv, ++lcount) {
-            const int rs = lcount % kRing;
-            if (!wait_bar(&ms->kv_empty[rs], ((lcount / kRing) & 1) ^ 1, ms, p.status)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(&ms->kv_full[rs], kTileBytes);
-            uint8_t *dst = ring + rs * kTileBytes;
-            const CUtensorMap *m = kv ? vm : km;
-            tma_load_3d(dst, m, 0, y, unit, &ms->kv_full[rs], policy_evict_first());
-            tma_load_3d(dst + kHalf, m, 64, y, unit, &ms->kv_full[rs], policy_evict_first());
-          }
-        }
-      }
-      ok = __shfl_sync(0xffffffffu, (int)ok, 0);
-      if (!ok) break;
     }
-    // Let issued copies land before the CTA can exit (after an abort).
-    if (lane == 0)
-      for (int j = max(0, lcount - kRing); j < lcount; ++j)
-        mbar_wait(&ms->kv_full[j % kRing], (j / kRing) & 1, nullptr, kWaitCycles / 4);
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -335,9 +354,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&ms->o_full[os]);
         return true;
       };
-      // Per item: S of tile j+1 is issued before P.V of tile j, so the
-      // softmax of one tile overlaps the score product of the next; the
-      // item's last P.V closes the item.
+      // S of tile u+1 is issued before P.V of tile u, also across items, so
+      // the softmax of one tile overlaps the score product of the next and
+      // an item's end does not stall the key stream. An item without tiles
+      // (empty or full cache) flushes the pending P.V first: the epilogue
+      // finishes items in order.
+      int pend = -1, pend_v = 0;  // tile waiting for its P.V, its value load
       for (int icount = 0; ok; ++icount) {
         const int slot = icount % kItemSlots;
         if (!wait_bar(&ms->item_full[slot], (icount / kItemSlots) & 1, ms, p.status)) break;
@@ -345,7 +367,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(&ms->item_empty[slot]);
         if (it >= total) break;
         const Item f = item_of(p, ms, it);
-        if (f.tiles == 0) continue;
+        if (f.tiles == 0) {
+          if (pend >= 0 && !pv(pend, pend_v)) break;
+          pend = -1;
+          continue;
+        }
         const int qs = qcount & 1;
         if (!wait_bar(&ms->q_full[qs], (qcount >> 1) & 1, ms, p.status)) break;
         ++qcount;
@@ -368,15 +394,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(&ms->kv_empty[ks]);
           mma_commit(&ms->s_full[ss]);
           lcount += 2;  // this tile's K and V loads
-          if (j > 0 && !pv(u - 1, lcount - 3)) {
+          if (pend >= 0 && !pv(pend, pend_v)) {
             ok = false;
             break;
           }
+          pend = u;
+          pend_v = lcount - 1;
         }
         if (!ok) break;
         mma_commit(&ms->q_empty[qs]);  // the item's queries are no longer read
-        if (!pv(u - 1, lcount - 1)) break;
       }
+      if (ok && pend >= 0) pv(pend, pend_v);
       mma_commit(&ms->mma_done);
       mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
     }
@@ -485,6 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (f.tiles > 0) combine(u - 1);
       // The new token, after the group's cache rows.
+      warp_wait(&ms->new_full[slot], (icount / kItemSlots) & 1, ms, p.status);
       if (f.chunk == f.nch - 1) {
         const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * 128;
         const float vn = __bfloat162float(((const __nv_bfloat16 *)p.v_new)[nb + i]);
@@ -522,6 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       named_bar_sync(1, 128);  // `last` read by all before it is written again
       if (last) {
         __threadfence();
+        if (i == 0) p.ctrl[2 + f.group] = 0;  // left at zero for the next call
 #pragma unroll
         for (int g = 0; g < G; ++g) {
           float mx = -INFINITY;
@@ -547,12 +577,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 256);
   }
-  // The last CTA to leave advances the lengths of the layers it appended to.
+  // The last CTA to leave advances the lengths of the layers it appended to
+  // and leaves the item and exit counters at zero for the next call.
   if (tid == 0) {
     __threadfence();
     if (atomicAdd(&p.ctrl[1], 1) == (int)gridDim.x - 1) {
       for (int t = 0; t < p.L; ++t)
         if (ms->len[t] >= 0) p.lens[p.order[t]] = ms->len[t] + 1;
+      p.ctrl[0] = 0;
+      p.ctrl[1] = 0;
     }
   }
 }
@@ -589,52 +622,124 @@ bool encode_cache(EncodeTiledFn enc, CUtensorMap *m, const void *base, int cap, 
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int sm_count() {
-  int dev = 0, n = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-  return n > 0 ? n : 1;
+constexpr int kMaxDevices = 64;
+
+int sm_count(int dev) {
+  static int n[kMaxDevices] = {};
+  if (dev < 0 || dev >= kMaxDevices) return 1;
+  if (n[dev] == 0) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    n[dev] = v > 0 ? v : 1;
+  }
+  return n[dev];
 }
 
 template <int G>
-cudaError_t launch_g(const TcDecParams &tp, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<G>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-  if (e != cudaSuccess) return e;
-  decode_tc_kernel<G><<<sm_count(), kThreads, kSmemBytes, st>>>(tp);
+cudaError_t launch_g(const TcDecParams &tp, int dev, cudaStream_t st) {
+  static bool attr_set[kMaxDevices] = {};
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  if (!attr_set[dev]) {
+    const cudaError_t e = cudaFuncSetAttribute(
+        decode_tc_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sm_count(dev));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, decode_tc_kernel<G>, tp);
   count_launches(1);
-  return cudaGetLastError();
+  return e;
+}
+
+// True when the tensor maps in `tp` already describe p's caches.
+bool same_caches(const TcDecParams &tp, int tp_dev, const DecParams &p, int dev) {
+  if (tp_dev != dev || tp.p.L != p.L || tp.p.B != p.B || tp.p.Hkv != p.Hkv) return false;
+  for (int t = 0; t < p.L; ++t) {
+    const int l = p.order[t];
+    if (tp.p.order[t] != l || tp.p.kc[l] != p.kc[l] || tp.p.vc[l] != p.vc[l] ||
+        tp.p.cap[l] != p.cap[l])
+      return false;
+  }
+  return true;
+}
+
+// Counter blocks this path left at zero, per device: the kernel resets its
+// counters on exit, so a workspace used by the previous call on the device
+// needs no clearing.
+struct CleanCtrl {
+  const void *ptr = nullptr;
+  size_t bytes = 0;
+};
+CleanCtrl g_clean[kMaxDevices];
+std::mutex g_clean_mu;
+
+cudaError_t clear_ctrl_if_needed(int dev, int *ctrl, size_t bytes, cudaStream_t st) {
+  std::lock_guard<std::mutex> lock(g_clean_mu);
+  CleanCtrl &c = g_clean[dev];
+  if (c.ptr == ctrl && c.bytes >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaMemsetAsync(ctrl, 0, bytes, st);
+  if (e == cudaSuccess) {
+    c.ptr = ctrl;
+    c.bytes = bytes;
+  }
+  return e;
 }
 
 }  // namespace
 
-bool decode_tc_supported(const ripple_decode_desc *d, int item_rows) {
+bool decode_tc_supported(const ripple_decode_desc *d) {
   const int G = d->n_q_heads / d->n_kv_heads;
   return d->dtype == RIPPLE_BF16 && d->head_dim == 128 && d->n_layers <= kTcMaxLayers &&
-         (G == 1 || G == 2 || G == 4 || G == 8) && item_rows == kTcItemRows &&
-         encode_fn() != nullptr;
+         (G == 1 || G == 2 || G == 4 || G == 8) && encode_fn() != nullptr;
 }
 
-cudaError_t launch_decode_tc(const DecParams &p, cudaStream_t st) {
+void decode_tc_forget_ctrl(const void *ctrl) {
+  std::lock_guard<std::mutex> lock(g_clean_mu);
+  for (auto &c : g_clean)
+    if (c.ptr == ctrl) c = CleanCtrl{};
+}
+
+cudaError_t launch_decode_tc(const DecParams &p, size_t ctrl_bytes, cudaStream_t st) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr || p.L > kTcMaxLayers) return cudaErrorNotSupported;
-  // Tensor maps by work-order position (the kernel indexes them that way).
-  static TcDecParams tp;  // large; filled under the lock, copied at launch
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  e = clear_ctrl_if_needed(dev, p.ctrl, ctrl_bytes, st);
+  if (e != cudaSuccess) return e;
+  // Tensor maps by work-order position (the kernel indexes them that way);
+  // re-encoded only when the caches change (serving loops reuse them).
+  static TcDecParams tp;  // large: kept off the stack, filled under the lock
+  static int tp_dev = -1;
   static std::mutex mu;
   std::lock_guard<std::mutex> lock(mu);
-  tp.p = p;
-  const int units = p.B * p.Hkv;
-  for (int t = 0; t < p.L; ++t) {
-    const int l = p.order[t];
-    if (!encode_cache(enc, &tp.kmap[t], p.kc[l], p.cap[l], units) ||
-        !encode_cache(enc, &tp.vmap[t], p.vc[l], p.cap[l], units))
-      return cudaErrorInvalidValue;
+  if (!same_caches(tp, tp_dev, p, dev)) {
+    tp_dev = -1;
+    const int units = p.B * p.Hkv;
+    for (int t = 0; t < p.L; ++t) {
+      const int l = p.order[t];
+      if (!encode_cache(enc, &tp.kmap[t], p.kc[l], p.cap[l], units) ||
+          !encode_cache(enc, &tp.vmap[t], p.vc[l], p.cap[l], units))
+        return cudaErrorInvalidValue;
+    }
+    tp_dev = dev;
   }
+  tp.p = p;
   switch (p.G) {
-    case 1: return launch_g<1>(tp, st);
-    case 2: return launch_g<2>(tp, st);
-    case 4: return launch_g<4>(tp, st);
-    case 8: return launch_g<8>(tp, st);
+    case 1: return launch_g<1>(tp, dev, st);
+    case 2: return launch_g<2>(tp, dev, st);
+    case 4: return launch_g<4>(tp, dev, st);
+    case 8: return launch_g<8>(tp, dev, st);
     default: return cudaErrorInvalidValue;
   }
 }

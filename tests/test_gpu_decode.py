@@ -66,10 +66,11 @@ DECODE_SHAPES = [
                           dtype="bf16", seed=42), [127, 513]),
     ("bf16-d64-G1", dict(n_layers=2, batch=2, n_q_heads=3, n_kv_heads=3, head_dim=64,
                          dtype="bf16", seed=43), [64, 200]),
-    # groups split over several 2048-row work items, item edges and a ragged tail
+    # groups split over several work items (4096 rows on the tensor-core path), item edges
+    # and a ragged tail
     ("bf16-d128-G4-split", dict(n_layers=4, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
                                 dtype="bf16", kv_dist="scaled_sinks", seed=47),
-     [2047, 2048, 2049, 4500]),
+     [2047, 4096, 4097, 8300]),
     ("bf16-d128-G1", dict(n_layers=2, batch=2, n_q_heads=2, n_kv_heads=2, head_dim=128,
                           dtype="bf16", seed=48), [0, 129]),
     ("bf16-d128-G2", dict(n_layers=2, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=128,
