@@ -211,10 +211,291 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
   }
 }
 
+// ---------------------------------------------------------------------------
+// The same selection spread over a cluster of kCluster CTAs per unit: CTA r
+// pools and keeps keys [r S, (r + 1) S) in its shared memory; per radix round
+// each CTA builds the histogram of its keys, and after a cluster barrier every
+// CTA reads all the cluster's histograms through distributed shared memory and
+// derives the same digit; the compaction offsets of a CTA are the counts of
+// the lower-ranked CTAs. Same result as select_kernel, bit for bit.
+
+constexpr int kCluster = 8;
+constexpr int kCThreads = 512;
+constexpr int kCWarps = kCThreads / 32;
+constexpr int kCMaxKeys = 40 * 1024;  // keys per CTA held in shared memory
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Shared::cluster address of the same shared-memory word in CTA `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(const void *p, uint32_t rank) {
+  uint32_t out;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(out) : "r"(smem_u32(p)), "r"(rank));
+  return out;
+}
+__device__ __forceinline__ uint4 ld_cluster_v4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared::cluster.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ uint2 ld_cluster_v2(uint32_t addr) {
+  uint2 v;
+  asm volatile("ld.shared::cluster.v2.u32 {%0, %1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Exclusive prefix sum of one int per thread over kCThreads threads.
+__device__ __forceinline__ int cta_exclusive_scan(int x, int *warp_tot, int *total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) warp_tot[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    const int t = lane < kCWarps ? warp_tot[lane] : 0;
+    int ti = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, ti, o);
+      if (lane >= o) ti += y;
+    }
+    if (lane < kCWarps) warp_tot[lane] = ti - t;
+    if (lane == 31) warp_tot[32] = ti;
+  }
+  __syncthreads();
+  const int res = warp_tot[wid] + incl - x;
+  *total = warp_tot[32];
+  __syncthreads();
+  return res;
+}
+
+__global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
+    select_cluster_kernel(LayerGeom g, const float *votes, int n_keep, int32_t *idx) {
+  extern __shared__ uint32_t sm[];
+  uint32_t *hist2 = sm;                            // [2][kBins], one per round parity
+  int *warp_tot = (int *)(sm + 2 * kBins);         // [33]
+  int *ctrl = warp_tot + 40;                       // [8]
+  int *cnt = ctrl + 8;                             // [2]: this CTA's (> tau, == tau) counts
+  int *wgt = cnt + 8, *weq = wgt + 32;             // [32] each
+  uint32_t *keys = sm + 2 * kBins + kCtrlWords;    // [S]
+
+  const uint32_t rank = cluster_rank();
+  const int unit = blockIdx.x / kCluster;
+  const int P = g.P, K = n_keep - g.W;
+  const int S = ((P + kCluster - 1) / kCluster + 31) & ~31;
+  const int k0 = min(P, (int)rank * S), k1 = min(P, k0 + S);
+  const float *v = votes + (size_t)unit * P;
+  int32_t *out = idx + (size_t)unit * n_keep;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+
+  if (rank == 0)
+    for (int j = tid; j < g.W; j += kCThreads) out[K + j] = P + j;
+  if (K <= 0) return;
+  if (K >= P) {
+    for (int t = k0 + tid; t < k1; t += kCThreads) out[t] = t;
+    return;
+  }
+
+  // This CTA's votes and the pooling halo, staged in shared memory with all
+  // loads in flight at once (one memory latency instead of one per step).
+  const int half = g.pool_kernel / 2;
+  const int lo = max(0, k0 - half), hi = min(P, k1 + half);
+  float *vs = reinterpret_cast<float *>(keys + S);  // [S + 2 * half]
+  {
+    constexpr int kU = 8;
+    for (int b0 = lo; b0 < hi; b0 += kU * kCThreads) {
+      float x[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int j = b0 + u * kCThreads + tid;
+        x[u] = j < hi ? __ldcg(v + j) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int j = b0 + u * kCThreads + tid;
+        if (j < hi) vs[j - lo] = x[u];
+      }
+    }
+  }
+  __syncthreads();
+  // Pooled keys of this CTA's range (the window reads across range edges).
+  const int step = 32 - 2 * half;
+  for (int seg = k0 + wid * step; seg < k1; seg += kCWarps * step) {
+    const int src = seg - half + lane;
+    const bool in = src >= 0 && src < P;
+    const float x = in ? vs[src - lo] : 0.f;
+    float r;
+    if (g.pool_type == RIPPLE_POOL_MAX) {
+      r = in ? x : -INFINITY;
+      const float own = r;
+      for (int d = 1; d <= half; ++d) {
+        r = fmaxf(r, __shfl_up_sync(0xffffffffu, own, d));
+        r = fmaxf(r, __shfl_down_sync(0xffffffffu, own, d));
+      }
+    } else if (g.pool_type == RIPPLE_POOL_AVG) {
+      float s = 0.f;
+      int c = 0;
+      for (int d = -half; d <= half; ++d) {
+        const float xv = d < 0 ? __shfl_up_sync(0xffffffffu, x, -d)
+                               : __shfl_down_sync(0xffffffffu, x, d);
+        const int pos = src + d;
+        if (pos >= 0 && pos < P) {
+          s = __fadd_rn(s, d == 0 ? x : xv);
+          ++c;
+        }
+      }
+      r = __fdiv_rn(s, (float)c);
+    } else {
+      r = x;
+    }
+    if (lane >= half && lane < 32 - half && src >= k0 && src < k1)
+      keys[src - k0] = order_key(r);
+  }
+  __syncthreads();
+
+  // Radix select of the K-th largest key over the whole unit.
+  uint32_t prefix = 0, mask = 0;
+  int remaining = K;
+  const int shifts[3] = {21, 10, 0};
+  const int widths[3] = {11, 11, 10};
+  const int n_local = k1 - k0;
+  for (int round = 0; round < 3; ++round) {
+    const int shift = shifts[round];
+    const uint32_t dmask = (1u << widths[round]) - 1u;
+    uint32_t *hist = hist2 + (round & 1) * kBins;
+    for (int i = tid; i < kBins; i += kCThreads) hist[i] = 0;
+    __syncthreads();
+    for (int base = 0; base < n_local; base += kCThreads) {
+      const int t = base + tid;
+      const uint32_t u = t < n_local ? keys[t] : 0u;
+      const bool hit = t < n_local && (u & mask) == prefix;
+      const uint32_t bin = hit ? (u >> shift) & dmask : 0xffffffffu;
+      const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+      if (hit && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+    }
+    cluster_sync_all();  // every CTA's histogram of this round is complete
+    // Thread j sums digits 2047-4j .. 2044-4j (descending) over the cluster:
+    // one 16-byte load from every CTA's histogram, all in flight together.
+    int c[4] = {0, 0, 0, 0};
+    const int d0 = kBins - 1 - 4 * tid;
+    {
+      uint4 h[kCluster];
+#pragma unroll
+      for (uint32_t r = 0; r < kCluster; ++r) h[r] = ld_cluster_v4(cluster_addr(hist + d0 - 3, r));
+#pragma unroll
+      for (uint32_t r = 0; r < kCluster; ++r) {
+        c[0] += (int)h[r].w;
+        c[1] += (int)h[r].z;
+        c[2] += (int)h[r].y;
+        c[3] += (int)h[r].x;
+      }
+    }
+    int total;
+    int above = cta_exclusive_scan(c[0] + c[1] + c[2] + c[3], warp_tot, &total);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (above < remaining && remaining <= above + c[q]) {
+        ctrl[0] = d0 - q;
+        ctrl[1] = remaining - above;
+      }
+      above += c[q];
+    }
+    __syncthreads();
+    prefix |= (uint32_t)ctrl[0] << shift;
+    mask |= dmask << shift;
+    remaining = ctrl[1];
+    __syncthreads();
+  }
+  const uint32_t tau = prefix;
+  const int take_eq = remaining;
+
+  // Ordered compaction over the cluster: counts per warp range, per CTA,
+  // then offsets from the lower-ranked CTAs.
+  const int per = ((n_local + kCWarps - 1) / kCWarps + 31) & ~31;
+  const int r0 = min(n_local, wid * per), r1 = min(n_local, r0 + per);
+  int cgt = 0, ceq = 0;
+  for (int b = r0; b < r1; b += 32) {
+    const int t = b + lane;
+    const uint32_t u = t < r1 ? keys[t] : 0u;
+    cgt += __popc(__ballot_sync(0xffffffffu, t < r1 && u > tau));
+    ceq += __popc(__ballot_sync(0xffffffffu, t < r1 && u == tau));
+  }
+  if (lane == 0) {
+    wgt[wid] = cgt;
+    weq[wid] = ceq;
+  }
+  __syncthreads();
+  if (wid == 0) {
+    const int a = lane < kCWarps ? wgt[lane] : 0, e = lane < kCWarps ? weq[lane] : 0;
+    int ia = a, ie = e;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int ya = __shfl_up_sync(0xffffffffu, ia, o), ye = __shfl_up_sync(0xffffffffu, ie, o);
+      if (lane >= o) {
+        ia += ya;
+        ie += ye;
+      }
+    }
+    if (lane < kCWarps) {
+      wgt[lane] = ia - a;
+      weq[lane] = ie - e;
+    }
+    if (lane == 31) {
+      cnt[0] = ia;
+      cnt[1] = ie;
+    }
+  }
+  cluster_sync_all();  // every CTA's counts are published
+  int gt_cta = 0, eq_cta = 0;
+  for (uint32_t r = 0; r < rank; ++r) {
+    const uint2 c = ld_cluster_v2(cluster_addr(cnt, r));
+    gt_cta += (int)c.x;
+    eq_cta += (int)c.y;
+  }
+  int gt_before = gt_cta + wgt[wid], eq_before = eq_cta + weq[wid];
+  const uint32_t below = (1u << lane) - 1u;
+  for (int b = r0; b < r1; b += 32) {
+    const int t = b + lane;
+    const uint32_t u = t < r1 ? keys[t] : 0u;
+    const bool gt = t < r1 && u > tau, eq = t < r1 && u == tau;
+    const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
+    const int g_rank = gt_before + __popc(bg & below);
+    const int e_rank = eq_before + __popc(be & below);
+    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = k0 + t;
+    gt_before += __popc(bg);
+    eq_before += __popc(be);
+  }
+  cluster_sync_all();  // no CTA leaves while others may still read its memory
+}
+
 }  // namespace
 
 cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
                           int n_keep, int32_t *idx, cudaStream_t st) {
+  const int per_cta = ((g.P + kCluster - 1) / kCluster + 31) & ~31;
+  if (per_cta <= kCMaxKeys && (long long)g.units * kCluster <= 0x7fffffff) {
+    // histograms, control words, keys, staged votes (with the pooling halo)
+    const size_t smem = sizeof(uint32_t) * (2 * kBins + kCtrlWords + 2 * per_cta + 32);
+    cudaError_t e = cudaFuncSetAttribute(select_cluster_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    select_cluster_kernel<<<g.units * kCluster, kCThreads, smem, st>>>(g, votes, n_keep, idx);
+    count_launches(1);
+    return cudaGetLastError();
+  }
   const int in_smem = g.P <= kSelectSmemKeys;
   const size_t smem = sizeof(uint32_t) * (kBins + kCtrlWords + (in_smem ? g.P : 0));
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
