@@ -111,9 +111,9 @@ extern "C" ripple_status ripple_compress_layer(const ripple_layer_desc *desc, in
   const bool keep_all = (n == g.T);
   float *votes = scores_out ? scores_out : ws.votes;
   if (g.P > 0 && (!keep_all || scores_out)) {
-    cudaError_t e = score_tc_supported(g)
-                        ? launch_score_tc(g, q_win, k, ws, votes, dev_status, st)
-                        : launch_score_simt(g, q_win, k, ws, votes, st);
+    cudaError_t e = score_tc1_supported(g)  ? launch_score_tc1(g, q_win, k, ws, votes, dev_status, st)
+                    : score_tc_supported(g) ? launch_score_tc(g, q_win, k, ws, votes, dev_status, st)
+                                            : launch_score_simt(g, q_win, k, ws, votes, st);
     RIPPLE_CUDA_TRY(e);
   }
   if (keep_all) {

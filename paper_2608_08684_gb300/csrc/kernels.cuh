@@ -44,6 +44,11 @@ bool score_tc_supported(const LayerGeom &g);
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
                             const CompressWs &ws, float *votes, int32_t *status,
                             cudaStream_t st);
+// Scoring with the window queries in TMEM (bf16, d = 128, G * w = 128 rows).
+bool score_tc1_supported(const LayerGeom &g);
+cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *k,
+                             const CompressWs &ws, float *votes, int32_t *status,
+                             cudaStream_t st);
 // Pooling + exact top-k per unit; writes idx [units][n].
 cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
                           int n_keep, int32_t *idx, cudaStream_t st);

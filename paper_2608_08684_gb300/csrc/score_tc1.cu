@@ -1,0 +1,614 @@
+// Observation-window token scoring for G * w = 128 window rows (SnapKV's rule
+// as RippleKV keeps it, Sec. 4.4, last paragraph), bf16, d = 128, on the
+// 5th-generation tensor cores with the window queries held in TMEM.
+//
+// Same work split as score_tc.cu (one persistent CTA per SM, item i on CTA
+// i mod grid, a publisher warp merging pass-1 row statistics), but each CTA's
+// step k runs P1(a_k) then P2(a_k-2), so keys are re-read from L2 two items
+// after their first read. Both passes compute
+// D[row][key] = Q . K_tile^T with the queries as the A operand in TMEM, so
+// shared memory holds only key tiles (a 6-stage ring) and each MMA reads only
+// its key tile from shared memory. Pass 2's vote of a key is a sum over rows,
+// i.e. over the epilogue threads: each warp reduce-scatters its 32 rows'
+// probabilities with shuffles (every lane ends with 4 keys' sums) and the
+// four warps' sums are added through shared memory.
+//
+// Warp roles (352 threads): warp 0 = key-tile producer, warp 1 = MMA issuer
+// and TMEM owner, warps 2-9 = two epilogue warpgroups taking alternate tiles
+// (they also stage each item's queries into TMEM, half of the columns each),
+// warp 10 = publisher of pass-1 results. Every wait is bounded; on timeout the
+// CTA raises RIPPLE_ETIMEOUT, every role leaves its loop and TMEM is released.
+#include <cuda.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc_ptx.cuh"
+
+namespace ripple {
+namespace {
+
+constexpr int kTile = 128;                      // keys per tile
+constexpr int kHalfBytes = kTile * 64 * 2;      // one TMA box: 64 dims of 128 keys
+constexpr int kTileBytes = 2 * kHalfBytes;
+constexpr int kThreads = 352;
+constexpr int kNK = 6;                          // key-tile stages
+constexpr int kLag = 2;                         // pass 2 of item k runs in step k + kLag
+constexpr int kNQ = kLag + 2;                   // query slots in TMEM (64 columns each)
+constexpr int kNA = 2;                          // accumulators in TMEM (128 columns each)
+constexpr int kPubSlots = 2;
+constexpr int kMinTilesPerItem = 8;
+constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then query slots
+constexpr long long kWaitCycles = 4000000000LL;
+
+struct Tc1Params {
+  int units, T, P, W, Hq, Hkv, G;
+  int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys)
+  int tpi, n_ch;           // key tiles per item, items per unit
+  int total_items;
+  float scale2;
+  const uint8_t *q;  // window queries [B][Hq][W][128] bf16
+  float2 *partial;   // [units][n_ch][128] (max, sum) per item and row, log2 domain
+  float *lognorm;    // [units][128]
+  float *votes;      // [units][P]
+  int *ctrl;         // [u] items of unit u published; [units + u] row statistics ready
+  int32_t *status;
+};
+
+struct ItemRef {
+  int unit, chunk;
+};
+
+__device__ __forceinline__ ItemRef item_of(const Tc1Params &p, int k) {
+  const int i = (int)blockIdx.x + k * (int)gridDim.x;
+  return {i / p.n_ch, i % p.n_ch};
+}
+
+__device__ __forceinline__ int items_of_cta(const Tc1Params &p) {
+  const int b = (int)blockIdx.x;
+  return b < p.total_items ? (p.total_items - 1 - b) / (int)gridDim.x + 1 : 0;
+}
+
+__device__ __forceinline__ void tiles_of(const Tc1Params &p, const ItemRef &it, int pass, int &t0,
+                                         int &t1) {
+  t0 = it.chunk * p.tpi;
+  t1 = min(pass == 1 ? p.n_tiles1 : p.n_tiles2, t0 + p.tpi);
+}
+
+// Step k of a CTA's schedule: pass 1 of its item k (if k < n), then pass 2
+// of its item k - kLag (if k >= kLag). A lag of two items leaves the other
+// CTAs a whole step to publish the row statistics pass 2 waits for; an
+// item's keys are re-read two items later (three items of keys per CTA in
+// L2). kZip takes the two passes' tiles in alternating pairs instead (a
+// steadier mix of DRAM and L2 reads per CTA; measured slower).
+constexpr bool kZip = false;
+
+struct Step {
+  int u1, a0, n1;  // pass 1: unit, first tile, tiles
+  int u2, b0, n2;  // pass 2
+  int len;         // max(n1, n2)
+};
+
+__device__ __forceinline__ Step step_of(const Tc1Params &p, int k, int n) {
+  Step s{0, 0, 0, 0, 0, 0, 0};
+  int e;
+  if (k < n) {
+    const ItemRef it = item_of(p, k);
+    tiles_of(p, it, 1, s.a0, e);
+    s.u1 = it.unit;
+    s.n1 = max(0, e - s.a0);
+  }
+  if (k >= kLag) {
+    const ItemRef it = item_of(p, k - kLag);
+    tiles_of(p, it, 2, s.b0, e);
+    s.u2 = it.unit;
+    s.n2 = max(0, e - s.b0);
+  }
+  s.len = s.n1 + s.n2;
+  return s;
+}
+
+// The epilogue warpgroup that takes the CTA's tile number `tc`: alternate
+// tiles, so that each warpgroup meets every phase of its accumulator slot.
+__device__ __forceinline__ int wg_of(int tc) { return tc & 1; }
+
+// Position j of step s's tile sequence: pass (1 or 2) and tile offset. With
+// kZip, tiles go in pairs P1 P1 P2 P2 P1 P1 ... (each warpgroup then gets
+// both kinds); the longer pass's remaining tiles follow.
+__device__ __forceinline__ void seq_at(const Step &s, int j, int &pass, int &idx) {
+  const int q = kZip ? min(s.n1, s.n2) / 2 : 0;  // pairs of each pass in the zipped part
+  if (j < 4 * q) {
+    const int blk = j >> 1;
+    pass = 1 + (blk & 1);
+    idx = ((blk >> 1) << 1) + (j & 1);
+    return;
+  }
+  j -= 4 * q;
+  const int r1 = s.n1 - 2 * q;
+  pass = j < r1 ? 1 : 2;
+  idx = 2 * q + (j < r1 ? j : j - r1);
+}
+
+struct Misc {
+  uint64_t k_full[kNK], k_empty[kNK], q_full[kNQ], q_empty[kNQ], acc_full[kNA], acc_empty[kNA];
+  uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
+  uint32_t tmem_base;
+  int abort_flag;
+  float2 pstat[kPubSlots][2][128];      // pass-1 row statistics per slot and warpgroup
+  alignas(16) float red[2][2][4][128];  // [warpgroup][tile parity][warp][key] vote partials
+};
+
+constexpr int kOffMisc = kNK * kTileBytes;
+constexpr int kSmemBytes = kOffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *ms,
+                                         int32_t *status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*(volatile int *)&ms->abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *(volatile int *)&ms->abort_flag = 1;
+      report(status, RIPPLE_ETIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ bool warp_wait(uint64_t *bar, uint32_t parity, Misc *ms,
+                                          int32_t *status) {
+  const bool ok = wait_bar(bar, parity, ms, status);
+  return __all_sync(0xffffffffu, ok);
+}
+
+__device__ __forceinline__ bool wait_ready(const int *flag, Misc *ms, int32_t *status) {
+  if (ld_acquire(flag)) return true;
+  const long long t0 = clock64();
+  for (;;) {
+    if (ld_acquire(flag)) return true;
+    if (*(volatile int *)&ms->abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *(volatile int *)&ms->abort_flag = 1;
+      report(status, RIPPLE_ETIMEOUT);
+      return false;
+    }
+    __nanosleep(64);
+  }
+}
+
+__device__ __forceinline__ void combine(float &m, float &l, float m2, float l2) {
+  const float mm = fmaxf(m, m2);
+  if (mm == -INFINITY) return;
+  l = l * fast_exp2(m - mm) + l2 * fast_exp2(m2 - mm);
+  m = mm;
+}
+
+// One reduce-scatter step over lanes `o` apart: of the 2n values, lanes with
+// bit `o` set keep the upper n, the others the lower n, each adding the
+// partner's copy of the half it keeps.
+template <int N>
+__device__ __forceinline__ void rs_step(float *v, int o, bool up) {
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    const float send = up ? v[i] : v[i + N];
+    const float keep = up ? v[i + N] : v[i];
+    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    score_tc1_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Tc1Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t *ktiles = smem;
+  Misc *ms = (Misc *)(smem + kOffMisc);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = items_of_cta(p);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kNK; ++i) {
+      mbar_init(&ms->k_full[i], 1);
+      mbar_init(&ms->k_empty[i], 1);
+    }
+    for (int i = 0; i < kNQ; ++i) {
+      mbar_init(&ms->q_full[i], 8);  // both warpgroups' four warps
+      mbar_init(&ms->q_empty[i], 1);
+    }
+    for (int i = 0; i < kNA; ++i) {
+      mbar_init(&ms->acc_full[i], 1);
+      mbar_init(&ms->acc_empty[i], 4);
+    }
+    for (int i = 0; i < kPubSlots; ++i) {
+      mbar_init(&ms->pub_full[i], 8);
+      mbar_init(&ms->pub_empty[i], 1);
+    }
+    mbar_init(&ms->mma_done, 1);
+    ms->abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&ms->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ms->tmem_base;
+
+  // Every role walks the same sequence of steps k = 0 .. n + kLag - 1.
+  if (warp == 0) {
+    // ------------------------------------------------ key-tile producer
+    if (lane == 0) {
+      int kcount = 0;
+      const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
+      bool ok = true;
+      for (int k = 0; k < n + kLag && ok; ++k) {
+        const Step st = step_of(p, k, n);
+        for (int j = 0; j < st.len && ok; ++j) {
+          {
+            int pass, s;
+            seq_at(st, j, pass, s);
+            const int unit = pass == 1 ? st.u1 : st.u2;
+            const int tt = pass == 1 ? st.a0 + s : st.b0 + s;
+            const int ks = kcount % kNK;
+            if (!wait_bar(&ms->k_empty[ks], ((kcount / kNK) & 1) ^ 1, ms, p.status)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
+            uint8_t *kb = ktiles + ks * kTileBytes;
+            const uint64_t pol = pass == 1 ? keep : drop;
+            tma_load_3d(kb, &kmap, 0, tt * kTile, unit, &ms->k_full[ks], pol);
+            tma_load_3d(kb + kHalfBytes, &kmap, 64, tt * kTile, unit, &ms->k_full[ks], pol);
+            ++kcount;
+          }
+        }
+      }
+      for (int j = max(0, kcount - kNK); j < kcount; ++j)
+        mbar_wait(&ms->k_full[j % kNK], (j / kNK) & 1, nullptr, kWaitCycles / 4);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int kcount = 0, acount = 0;
+      constexpr uint32_t id = idesc_bf16(128, 128);
+      const uint32_t kbase = smem_u32(ktiles);
+      bool ok = true;
+      for (int k = 0; k < n + kLag && ok; ++k) {
+        const Step st = step_of(p, k, n);
+        const int qs1 = k % kNQ, qs2 = (k + kNQ - kLag) % kNQ;
+        if (k < n && !wait_bar(&ms->q_full[qs1], (k / kNQ) & 1, ms, p.status)) break;
+        for (int j = 0; j < st.len && ok; ++j) {
+          {
+            int pass, s;
+            seq_at(st, j, pass, s);
+            const uint32_t qa = tmem + kQCol + (pass == 1 ? qs1 : qs2) * 64;
+            const int ks = kcount % kNK, as = acount % kNA;
+            if (!wait_bar(&ms->k_full[ks], (kcount / kNK) & 1, ms, p.status) ||
+                !wait_bar(&ms->acc_empty[as], ((acount / kNA) & 1) ^ 1, ms, p.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t d = tmem + as * 128;
+            const uint32_t ka = kbase + ks * kTileBytes;
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16_tmem_a(d, qa + kk * 8,
+                              sw128_desc(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32), id, kk > 0);
+            mma_commit(&ms->k_empty[ks]);
+            mma_commit(&ms->acc_full[as]);
+            ++kcount;
+            ++acount;
+          }
+        }
+        if (ok && k >= kLag) mma_commit(&ms->q_empty[qs2]);  // item k - kLag's slot is free
+      }
+      mma_commit(&ms->mma_done);
+      mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
+    }
+  } else if (warp == 10) {
+    // ------------------------------------------------ publisher of pass-1 results
+    for (int k = 0; k < n; ++k) {
+      const int slot = k % kPubSlots;
+      if (!warp_wait(&ms->pub_full[slot], (k / kPubSlots) & 1, ms, p.status)) break;
+      const ItemRef it = item_of(p, k);
+      float2 *mine = p.partial + ((size_t)it.unit * p.n_ch + it.chunk) * 128;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int r = lane + 32 * j;
+        float2 a = ms->pstat[slot][0][r];
+        const float2 b = ms->pstat[slot][1][r];
+        combine(a.x, a.y, b.x, b.y);
+        mine[r] = a;
+      }
+      __syncwarp();
+      int last = 0;
+      if (lane == 0) {
+        mbar_arrive(&ms->pub_empty[slot]);
+        __threadfence();
+        last = atomicAdd(&p.ctrl[it.unit], 1) == p.n_ch - 1;
+      }
+      last = __shfl_sync(0xffffffffu, last, 0);
+      if (last) {
+        __threadfence();
+        const float2 *part = p.partial + (size_t)it.unit * p.n_ch * 128;
+        float mm[4], ll[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          mm[j] = -INFINITY;
+          ll[j] = 0.f;
+        }
+        for (int c0 = 0; c0 < p.n_ch; c0 += 8) {
+          float2 q[8][4];
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              q[c][j] = c0 + c < p.n_ch ? __ldcg(&part[(size_t)(c0 + c) * 128 + lane + 32 * j])
+                                        : make_float2(-INFINITY, 0.f);
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) combine(mm[j], ll[j], q[c][j].x, q[c][j].y);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          p.lognorm[(size_t)it.unit * 128 + lane + 32 * j] = mm[j] + __log2f(ll[j]);
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release(&p.ctrl[p.units + it.unit], 1);
+      }
+    }
+  } else {
+    // ------------------------------------------------ epilogue warpgroups
+    const int wg = (warp - 2) >> 2;
+    const int quarter = warp & 3;              // TMEM lanes this warp may access
+    const int r = quarter * 32 + lane;         // window row of this thread
+    const int wtid = threadIdx.x - 64 - wg * 128;
+    const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
+    int tcount = 0, wcount = 0;  // tiles seen, tiles this warpgroup took
+
+    // Stages item k's window queries into query slot k % kNQ: this thread's
+    // row, this warpgroup's half of the 64 columns.
+    auto load_q = [&](int k) {
+      const int qs = k % kNQ;
+      warp_wait(&ms->q_empty[qs], ((k / kNQ) & 1) ^ 1, ms, p.status);
+      tc_fence_after();
+      const ItemRef it = item_of(p, k);
+      const int b = it.unit / p.Hkv, h = it.unit % p.Hkv;
+      const size_t row = (size_t)(b * p.Hq + h * p.G) * p.W + r;
+      const uint4 *src = reinterpret_cast<const uint4 *>(p.q + row * 256 + wg * 128);
+      uint32_t w[32];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const uint4 u = __ldg(src + c);
+        w[4 * c] = u.x;
+        w[4 * c + 1] = u.y;
+        w[4 * c + 2] = u.z;
+        w[4 * c + 3] = u.w;
+      }
+      tmem_st32(tmem + lane_addr + kQCol + qs * 64 + wg * 32, w);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ms->q_full[qs]);
+    };
+
+    if (n > 0) load_q(0);
+    // Inside an item every warp follows the same control flow even if a wait
+    // gives up (the tile is then skipped), so that the named barriers below
+    // are always reached by all of their threads.
+    for (int k = 0; k < n + kLag; ++k) {
+      if (k + 1 < n) load_q(k + 1);
+      const Step st = step_of(p, k, n);
+      float m = -INFINITY, l = 0.f;    // pass 1 of item k: this row's max and sum
+      const int last_vis = p.P + r % p.W;
+      float off = 0.f;                 // pass 2 of item k - kLag: this row's log-normaliser
+      for (int j = 0; j < st.len; ++j) {
+        int pass, s;
+        seq_at(st, j, pass, s);
+        if (pass == 1) {
+          // ---------------- a pass-1 tile of item k
+          const int t = st.a0 + s;
+          const int mine = wg_of(tcount) == wg;
+          const int as = tcount % kNA, ph = (tcount / kNA) & 1;
+          ++tcount;
+          if (mine && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
+            tc_fence_after();
+            uint32_t x[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + as * 128 + c * 32, x[c]);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+            if ((t + 1) * kTile - 1 >= p.P) {  // keys this row cannot see -> -inf
+#pragma unroll
+              for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (t * kTile + c * 32 + j > last_vis) x[c][j] = 0xff800000u;
+            }
+            float mx[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) mx[i] = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+              for (int j = 0; j < 32; ++j) mx[j & 7] = fmaxf(mx[j & 7], __uint_as_float(x[c][j]));
+            const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                     fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+            if (tmax != -INFINITY) {
+              const float mnew = fmaxf(m, tmax * p.scale2);
+              float sv[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) sv[i] = 0.f;
+#pragma unroll
+              for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  sv[j & 7] += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
+              const float sum =
+                  ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
+              l = l * fast_exp2(m - mnew) + sum;
+              m = mnew;
+            }
+          }
+          if (s == st.n1 - 1) {
+            // Item k's last pass-1 tile: this warpgroup's row statistics go to
+            // the publisher now, ahead of the step's pass-2 tiles.
+            const int slot = k % kPubSlots;
+            warp_wait(&ms->pub_empty[slot], ((k / kPubSlots) & 1) ^ 1, ms, p.status);
+            ms->pstat[slot][wg][r] = make_float2(m, l);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ms->pub_full[slot]);
+          }
+        }
+        if (pass == 2) {
+          // ---------------- a pass-2 tile of item k - kLag: votes of its keys
+          if (s == 0) {
+            if (wtid == 0) wait_ready(&p.ctrl[p.units + st.u2], ms, p.status);
+            named_bar_sync(3 + wg, 128);
+            off = __ldcg(&p.lognorm[(size_t)st.u2 * 128 + r]);
+          }
+          const int t = st.b0 + s;
+          const int mine = wg_of(tcount) == wg;
+          const int as = tcount % kNA, ph = (tcount / kNA) & 1;
+          ++tcount;
+          if (mine) {
+            const bool got = warp_wait(&ms->acc_full[as], ph, ms, p.status);
+            float v[128];
+            if (got) {
+              tc_fence_after();
+              uint32_t x[4][32];
+#pragma unroll
+              for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + as * 128 + c * 32, x[c]);
+              tmem_wait_ld();
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+#pragma unroll
+              for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  v[c * 32 + j] = fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -off));
+            } else {
+#pragma unroll
+              for (int j = 0; j < 128; ++j) v[j] = 0.f;
+            }
+            // Sum over the warp's 32 rows: lane L ends with keys 4L .. 4L + 3.
+            rs_step<64>(v, 16, lane & 16);
+            rs_step<32>(v, 8, lane & 8);
+            rs_step<16>(v, 4, lane & 4);
+            rs_step<8>(v, 2, lane & 2);
+            rs_step<4>(v, 1, lane & 1);
+            float *red = ms->red[wg][wcount & 1][0];
+            *reinterpret_cast<float4 *>(red + quarter * 128 + 4 * lane) =
+                make_float4(v[0], v[1], v[2], v[3]);
+            named_bar_sync(3 + wg, 128);
+            const float vote =
+                (red[wtid] + red[128 + wtid]) + (red[256 + wtid] + red[384 + wtid]);
+            const int key = t * kTile + wtid;
+            if (key < p.P) p.votes[(size_t)st.u2 * p.P + key] = vote;
+            ++wcount;
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncwarp();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------------------------------ host side
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn == nullptr) {
+    void *ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (EncodeTiledFn)ptr;
+  }
+  return fn;
+}
+
+}  // namespace
+
+bool score_tc1_supported(const LayerGeom &g) {
+  return g.dtype == RIPPLE_BF16 && g.D == 128 && g.R == 128 && g.P > 0 && encode_fn() != nullptr;
+}
+
+cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *k,
+                             const CompressWs &ws, float *votes, int32_t *status,
+                             cudaStream_t st) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  CUtensorMap kmap;
+  {
+    cuuint64_t dims[3] = {128, (cuuint64_t)g.T, (cuuint64_t)g.units};
+    cuuint64_t strides[2] = {256, (cuuint64_t)g.T * 256};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k), dims, strides, box,
+            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (sms <= 0) sms = 1;
+  Tc1Params p;
+  p.units = g.units;
+  p.T = g.T;
+  p.P = g.P;
+  p.W = g.W;
+  p.Hq = g.Hq;
+  p.Hkv = g.Hkv;
+  p.G = g.G;
+  p.n_tiles1 = (g.T + kTile - 1) / kTile;
+  p.n_tiles2 = (g.P + kTile - 1) / kTile;
+  // At least kMinTilesPerItem tiles per item, and no more items per unit than
+  // SMs (the deadlock-free schedule needs <= 2x as many as CTAs).
+  const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
+  p.tpi = tpi_min > kMinTilesPerItem ? tpi_min : kMinTilesPerItem;
+  p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
+  p.total_items = g.units * p.n_ch;
+  p.scale2 = g.scale2;
+  p.q = (const uint8_t *)q_win;
+  p.partial = ws.row_partial;
+  p.lognorm = ws.row_lognorm;
+  p.votes = votes;
+  p.ctrl = ws.counters;
+  p.status = status;
+  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * g.units, st);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(score_tc1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kSmemBytes);
+  if (e != cudaSuccess) return e;
+  const int grid = p.total_items < sms ? p.total_items : sms;
+  void *args[] = {(void *)&kmap, (void *)&p};
+  e = cudaLaunchCooperativeKernel((const void *)score_tc1_kernel, dim3(grid), dim3(kThreads), args,
+                                  (size_t)kSmemBytes, st);
+  count_launches(1);
+  return e;
+}
+
+}  // namespace ripple
