@@ -262,13 +262,16 @@ class Serving:
             self.v.append(synth.layer_values(wl, layer, device))
         self.desc = R.layer_desc(B, Hq, Hkv, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
                                  wl.torch_dtype)
-        self.ws = torch.empty(R.ripple_compress_workspace_bytes(self.desc), dtype=torch.uint8,
-                              device=device)
+        # one call compresses every layer (ripple_compress_layers)
+        self.ws = torch.empty(R.ripple_compress_layers_workspace_bytes(self.desc, L),
+                              dtype=torch.uint8, device=device)
         self.k_out = [torch.zeros(B, Hkv, c, d, dtype=wl.torch_dtype, device=device)
                       for c in self.caps]
         self.v_out = [torch.zeros_like(t) for t in self.k_out]
         self.idx = [torch.empty(B * Hkv * n, dtype=torch.int32, device=device)
                     for n in self.n_keep]
+        self.ctables = R.CompressTables(self.q_win, self.k, self.v, self.k_out, self.v_out,
+                                        self.idx)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
         self.dq, self.dk, self.dv = [], [], []
         for t in range(wl.decode_steps):
@@ -294,11 +297,9 @@ class Serving:
         if timers:
             c0 = ev()
             c0.record()
-        for layer in range(wl.n_layers):
-            n = R.ripple_compress_layer(self.desc, budgets[layer], self.q_win[layer], self.k[layer],
-                                        self.v[layer], self.k_out[layer], self.v_out[layer],
-                                        self.idx[layer], self.ws, dev_status=self.status)
-            assert n == self.n_keep[layer]
+        n = R.ripple_compress_layers(self.desc, budgets, self.ctables, self.ws,
+                                     dev_status=self.status)
+        assert n == self.n_keep
         if timers:
             c1 = ev()
             c1.record()

@@ -163,6 +163,43 @@ ripple_status ripple_compress_layer(const ripple_layer_desc *desc, int64_t budge
                                     size_t workspace_bytes, int32_t *dev_status,
                                     void *stream);
 
+/* Layers one ripple_compress_layers call may cover. */
+#define RIPPLE_COMPRESS_MAX_LAYERS 80
+
+/* Device workspace bytes ripple_compress_layers needs for n_layers layers of
+ * this shape. */
+ripple_status ripple_compress_layers_workspace_bytes(const ripple_layer_desc *desc,
+                                                     int32_t n_layers, size_t *bytes_host);
+
+/*
+ * ripple_compress_layers -- ripple_compress_layer for n_layers layers of the
+ * same shape (same desc) in one call, each with its own budget (the budgets
+ * b_l of Eqs. 9-12). Layer l's result is exactly that of ripple_compress_layer
+ * with budgets_host[l] and layer l's buffers; the layers are processed
+ * together (bf16, d = 128, G * w = 128: three launches for all layers, so the
+ * GPU is not idle between layers), otherwise one after another.
+ *
+ * n_layers     1..RIPPLE_COMPRESS_MAX_LAYERS, and n_layers * B * Hkv <= 65535
+ * budgets_host host [n_layers]
+ * q_win_host, k_host, v_host, k_out_host, v_out_host, idx_out_host
+ *              host arrays of n_layers device pointers with the layouts of
+ *              ripple_compress_layer (idx_out_host[l]: [B][Hkv][n_l] int32)
+ * caps_host    host [n_layers]: rows per (b, h) of each layer's outputs
+ * n_keep_host  host [n_layers], out: n_l of every layer
+ * workspace    device scratch of at least
+ *              ripple_compress_layers_workspace_bytes(desc, n_layers) bytes,
+ *              256-byte aligned, no initialisation needed
+ * Errors: RIPPLE_EINVAL (as ripple_compress_layer, for any layer),
+ * RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status as ripple_compress_layer.
+ */
+ripple_status ripple_compress_layers(const ripple_layer_desc *desc, int32_t n_layers,
+                                     const int64_t *budgets_host, const void *const *q_win_host,
+                                     const void *const *k_host, const void *const *v_host,
+                                     void *const *k_out_host, void *const *v_out_host,
+                                     const int32_t *caps_host, int32_t *const *idx_out_host,
+                                     int32_t *n_keep_host, void *workspace,
+                                     size_t workspace_bytes, int32_t *dev_status, void *stream);
+
 /*
  * ripple_select_layer -- steps 2-4 of ripple_compress_layer (pooling, top-k
  * selection with the window appended, gather) from caller-provided votes

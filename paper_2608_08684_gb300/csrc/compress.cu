@@ -111,7 +111,7 @@ extern "C" ripple_status ripple_compress_layer(const ripple_layer_desc *desc, in
   const bool keep_all = (n == g.T);
   float *votes = scores_out ? scores_out : ws.votes;
   if (g.P > 0 && (!keep_all || scores_out)) {
-    cudaError_t e = score_tc1_supported(g)  ? launch_score_tc1(g, q_win, k, ws, votes, dev_status, st)
+    cudaError_t e = score_tc1_supported(g)  ? launch_score_tc1(g, 1, &q_win, &k, ws, votes, dev_status, st)
                     : score_tc_supported(g) ? launch_score_tc(g, q_win, k, ws, votes, dev_status, st)
                                             : launch_score_simt(g, q_win, k, ws, votes, st);
     RIPPLE_CUDA_TRY(e);
@@ -119,9 +119,9 @@ extern "C" ripple_status ripple_compress_layer(const ripple_layer_desc *desc, in
   if (keep_all) {
     RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
   } else {
-    RIPPLE_CUDA_TRY(launch_select(g, votes, ws, n, idx_out, st));
+    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, st));
   }
-  RIPPLE_CUDA_TRY(launch_gather(g, k, v, idx_out, n, k_out, v_out, cap, dev_status, st));
+  RIPPLE_CUDA_TRY(launch_gather(g, 1, &k, &v, &idx_out, &n, &k_out, &v_out, &cap, dev_status, st));
   *n_keep_host = n;
   return RIPPLE_OK;
 }
@@ -149,9 +149,89 @@ extern "C" ripple_status ripple_select_layer(const ripple_layer_desc *desc, int6
   if (n == g.T) {
     RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
   } else {
-    RIPPLE_CUDA_TRY(launch_select(g, votes, ws, n, idx_out, st));
+    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, st));
   }
-  RIPPLE_CUDA_TRY(launch_gather(g, k, v, idx_out, n, k_out, v_out, cap, dev_status, st));
+  RIPPLE_CUDA_TRY(launch_gather(g, 1, &k, &v, &idx_out, &n, &k_out, &v_out, &cap, dev_status, st));
   *n_keep_host = n;
+  return RIPPLE_OK;
+}
+
+// Workspace of a multi-layer call: the single-layer carve-up for all layers'
+// units at once (votes [n_layers][units][P] contiguous).
+static CompressWs carve_layers_ws(const LayerGeom &g, int n_layers, void *base) {
+  LayerGeom all = g;
+  all.units = g.units * n_layers;
+  return carve_compress_ws(all, base);
+}
+
+extern "C" ripple_status ripple_compress_layers_workspace_bytes(const ripple_layer_desc *desc,
+                                                                int32_t n_layers,
+                                                                size_t *bytes_host) {
+  LayerGeom g;
+  if (!make_geom(desc, &g) || bytes_host == nullptr || n_layers < 1 ||
+      n_layers > RIPPLE_COMPRESS_MAX_LAYERS || (int64_t)g.units * n_layers > 65535)
+    return RIPPLE_EINVAL;
+  *bytes_host = carve_layers_ws(g, n_layers, nullptr).bytes;
+  return RIPPLE_OK;
+}
+
+extern "C" ripple_status ripple_compress_layers(
+    const ripple_layer_desc *desc, int32_t n_layers, const int64_t *budgets_host,
+    const void *const *q_win_host, const void *const *k_host, const void *const *v_host,
+    void *const *k_out_host, void *const *v_out_host, const int32_t *caps_host,
+    int32_t *const *idx_out_host, int32_t *n_keep_host, void *workspace, size_t workspace_bytes,
+    int32_t *dev_status, void *stream) {
+  LayerGeom g;
+  if (!make_geom(desc, &g) || n_layers < 1 || n_layers > RIPPLE_COMPRESS_MAX_LAYERS ||
+      (int64_t)g.units * n_layers > 65535)
+    return RIPPLE_EINVAL;
+  if (!budgets_host || !q_win_host || !k_host || !v_host || !k_out_host || !v_out_host ||
+      !caps_host || !idx_out_host || !n_keep_host || !workspace || ((uintptr_t)workspace & 255u))
+    return RIPPLE_EINVAL;
+  auto aligned = [](const void *p) { return p != nullptr && ((uintptr_t)p & 15u) == 0; };
+  int n[RIPPLE_COMPRESS_MAX_LAYERS];
+  int cap[RIPPLE_COMPRESS_MAX_LAYERS];
+  for (int l = 0; l < n_layers; ++l) {
+    if (budgets_host[l] < 0 || !aligned(q_win_host[l]) || !aligned(k_host[l]) ||
+        !aligned(v_host[l]) || !aligned(k_out_host[l]) || !aligned(v_out_host[l]) ||
+        !aligned(idx_out_host[l]))
+      return RIPPLE_EINVAL;
+    n[l] = ripple_keep_count(budgets_host[l], g.T, g.W);
+    cap[l] = caps_host[l];
+    if (n[l] < 0 || cap[l] < n[l]) return RIPPLE_EINVAL;
+  }
+  const CompressWs ws = carve_layers_ws(g, n_layers, workspace);
+  if (workspace_bytes < ws.bytes) return RIPPLE_EWORKSPACE;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (g.P > 0 && score_tc1_supported(g)) {
+    // All layers in three launches: scoring, selection, gather.
+    RIPPLE_CUDA_TRY(launch_score_tc1(g, n_layers, q_win_host, k_host, ws, ws.votes, dev_status,
+                                     st));
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, st));
+    RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
+                                  (const int32_t *const *)idx_out_host, n, k_out_host,
+                                  v_out_host, cap, dev_status, st));
+  } else {
+    // Other shapes: layer by layer (one layer's share of the workspace each).
+    const CompressWs one = carve_compress_ws(g, workspace);
+    for (int l = 0; l < n_layers; ++l) {
+      const bool keep_all = n[l] == g.T;
+      if (g.P > 0 && !keep_all) {
+        cudaError_t e =
+            score_tc_supported(g)
+                ? launch_score_tc(g, q_win_host[l], k_host[l], one, one.votes, dev_status, st)
+                : launch_score_simt(g, q_win_host[l], k_host[l], one, one.votes, st);
+        RIPPLE_CUDA_TRY(e);
+      }
+      int32_t *idx = idx_out_host[l];
+      if (keep_all)
+        RIPPLE_CUDA_TRY(launch_iota(g, idx, st));
+      else
+        RIPPLE_CUDA_TRY(launch_select(g, 1, one.votes, one, &n[l], &idx, st));
+      RIPPLE_CUDA_TRY(launch_gather(g, 1, &k_host[l], &v_host[l], &idx_out_host[l], &n[l],
+                                    &k_out_host[l], &v_out_host[l], &cap[l], dev_status, st));
+    }
+  }
+  for (int l = 0; l < n_layers; ++l) n_keep_host[l] = n[l];
   return RIPPLE_OK;
 }

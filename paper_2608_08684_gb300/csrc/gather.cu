@@ -16,15 +16,31 @@ namespace {
 constexpr int kTileRows = 64;
 constexpr int kThreads = 64;
 
-__global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t *k, const uint8_t *v,
-                                                          const int32_t *idx, int T, int n_keep,
-                                                          int row_bytes, uint8_t *k_out,
-                                                          uint8_t *v_out, int cap,
+// Layers of one launch: units per layer, and per layer the input caches
+// [upl][T][d], the kept indices [upl][n_keep], the outputs [upl][cap][d].
+struct GatherTable {
+  int upl;
+  const uint8_t *k[kCompressMaxLayers];
+  const uint8_t *v[kCompressMaxLayers];
+  const int32_t *idx[kCompressMaxLayers];
+  uint8_t *k_out[kCompressMaxLayers];
+  uint8_t *v_out[kCompressMaxLayers];
+  int n_keep[kCompressMaxLayers];
+  int cap[kCompressMaxLayers];
+};
+
+__global__ void __launch_bounds__(kThreads) gather_kernel(const __grid_constant__ GatherTable tab,
+                                                          int T, int row_bytes,
                                                           int32_t *status) {
   extern __shared__ __align__(128) uint8_t tile[];
   __shared__ __align__(8) uint64_t bar;
-  const int unit = blockIdx.y;
+  const int layer = blockIdx.y / tab.upl, unit = blockIdx.y % tab.upl;
+  const int n_keep = tab.n_keep[layer], cap = tab.cap[layer];
+  const uint8_t *k = tab.k[layer], *v = tab.v[layer];
+  uint8_t *k_out = tab.k_out[layer], *v_out = tab.v_out[layer];
+  const int32_t *idx = tab.idx[layer];
   const int j0 = blockIdx.x * kTileRows;
+  if (j0 >= n_keep) return;  // this layer keeps fewer rows than the longest one
   const int rows = min(kTileRows, n_keep - j0);
   uint8_t *tk = tile;
   uint8_t *tv = tile + (size_t)kTileRows * row_bytes;
@@ -62,18 +78,34 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const uint8_t *k, cons
 
 }  // namespace
 
-cudaError_t launch_gather(const LayerGeom &g, const void *k, const void *v, const int32_t *idx,
-                          int n_keep, void *k_out, void *v_out, int cap, int32_t *status,
-                          cudaStream_t st) {
+cudaError_t launch_gather(const LayerGeom &g, int n_layers, const void *const *k,
+                          const void *const *v, const int32_t *const *idx, const int *n_keep,
+                          void *const *k_out, void *const *v_out, const int *cap,
+                          int32_t *status, cudaStream_t st) {
+  if (n_layers < 1 || n_layers > kCompressMaxLayers ||
+      (long long)g.units * n_layers > 65535)
+    return cudaErrorInvalidValue;
+  GatherTable tab;
+  tab.upl = g.units;
+  int max_keep = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    tab.k[l] = (const uint8_t *)k[l];
+    tab.v[l] = (const uint8_t *)v[l];
+    tab.idx[l] = idx[l];
+    tab.k_out[l] = (uint8_t *)k_out[l];
+    tab.v_out[l] = (uint8_t *)v_out[l];
+    tab.n_keep[l] = n_keep[l];
+    tab.cap[l] = cap[l];
+    max_keep = n_keep[l] > max_keep ? n_keep[l] : max_keep;
+  }
+  if (max_keep == 0) return cudaSuccess;
   const int row_bytes = g.D * (g.dtype == RIPPLE_F32 ? 4 : 2);
   const size_t smem = (size_t)2 * kTileRows * row_bytes;
   cudaError_t e = cudaFuncSetAttribute(gather_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid((n_keep + kTileRows - 1) / kTileRows, g.units);
-  gather_kernel<<<grid, kThreads, smem, st>>>((const uint8_t *)k, (const uint8_t *)v, idx, g.T,
-                                              n_keep, row_bytes, (uint8_t *)k_out,
-                                              (uint8_t *)v_out, cap, status);
+  const dim3 grid((max_keep + kTileRows - 1) / kTileRows, g.units * n_layers);
+  gather_kernel<<<grid, kThreads, smem, st>>>(tab, g.T, row_bytes, status);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -21,6 +21,9 @@ struct LayerGeom {
   float scale2;                       // logit scale * log2(e)
 };
 
+// Layers one multi-layer compression call covers.
+constexpr int kCompressMaxLayers = RIPPLE_COMPRESS_MAX_LAYERS;
+
 constexpr int kScoreChunk = 128;      // keys per scoring work item
 constexpr int kSelectThreads = 1024;  // threads of the selection CTA
 constexpr int kSelectSmemKeys = 48 * 1024;  // prefix lengths up to this keep keys in smem
@@ -44,19 +47,24 @@ bool score_tc_supported(const LayerGeom &g);
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
                             const CompressWs &ws, float *votes, int32_t *status,
                             cudaStream_t st);
-// Scoring with the window queries in TMEM (bf16, d = 128, G * w = 128 rows).
+// Scoring with the window queries in TMEM (bf16, d = 128, G * w = 128 rows),
+// for n_layers layers of the same shape in one launch; ws is carved for
+// n_layers * g.units units and votes is [n_layers][g.units][P].
 bool score_tc1_supported(const LayerGeom &g);
-cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *k,
-                             const CompressWs &ws, float *votes, int32_t *status,
-                             cudaStream_t st);
-// Pooling + exact top-k per unit; writes idx [units][n].
-cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
-                          int n_keep, int32_t *idx, cudaStream_t st);
+cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const *q_win,
+                             const void *const *k, const CompressWs &ws, float *votes,
+                             int32_t *status, cudaStream_t st);
+// Pooling + exact top-k per unit of n_layers layers (votes [n_layers][units][P]);
+// writes idx[l] [units][n_keep[l]].
+cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
+                          const CompressWs &ws, const int *n_keep, int32_t *const *idx,
+                          cudaStream_t st);
 // idx = 0..T-1 for every unit (keep-all case).
 cudaError_t launch_iota(const LayerGeom &g, int32_t *idx, cudaStream_t st);
-// Gather kept K and V rows into [units][cap][d].
-cudaError_t launch_gather(const LayerGeom &g, const void *k, const void *v, const int32_t *idx,
-                          int n_keep, void *k_out, void *v_out, int cap, int32_t *status,
-                          cudaStream_t st);
+// Gather kept K and V rows of n_layers layers into [units][cap[l]][d].
+cudaError_t launch_gather(const LayerGeom &g, int n_layers, const void *const *k,
+                          const void *const *v, const int32_t *const *idx, const int *n_keep,
+                          void *const *k_out, void *const *v_out, const int *cap,
+                          int32_t *status, cudaStream_t st);
 
 }  // namespace ripple

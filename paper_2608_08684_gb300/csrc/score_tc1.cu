@@ -21,6 +21,8 @@
 #include <cuda.h>
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc_ptx.cuh"
@@ -42,15 +44,15 @@ constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then quer
 constexpr long long kWaitCycles = 4000000000LL;
 
 struct Tc1Params {
-  int units, T, P, W, Hq, Hkv, G;
+  int units, upl, T, P, W, Hq, Hkv, G;  // units of all layers, units per layer
   int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys)
   int tpi, n_ch;           // key tiles per item, items per unit
   int total_items;
   float scale2;
-  const uint8_t *q;  // window queries [B][Hq][W][128] bf16
+  const uint8_t *q[kCompressMaxLayers];  // per layer: window queries [B][Hq][W][128] bf16
   float2 *partial;   // [units][n_ch][128] (max, sum) per item and row, log2 domain
   float *lognorm;    // [units][128]
-  float *votes;      // [units][P]
+  float *votes;      // [units][P], layer-major
   int *ctrl;         // [u] items of unit u published; [units + u] row statistics ready
   int32_t *status;
 };
@@ -200,8 +202,16 @@ __device__ __forceinline__ void rs_step(float *v, int o, bool up) {
   }
 }
 
+// Kernel argument: the keys of every layer as 3-D tensor maps [unit][T][128],
+// and the parameters.
+struct Tc1Launch {
+  CUtensorMap kmap[kCompressMaxLayers];
+  Tc1Params p;
+};
+
 __global__ void __launch_bounds__(kThreads, 1)
-    score_tc1_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ Tc1Params p) {
+    score_tc1_kernel(const __grid_constant__ Tc1Launch lp) {
+  const Tc1Params &p = lp.p;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ktiles = smem;
@@ -262,8 +272,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
             uint8_t *kb = ktiles + ks * kTileBytes;
             const uint64_t pol = pass == 1 ? keep : drop;
-            tma_load_3d(kb, &kmap, 0, tt * kTile, unit, &ms->k_full[ks], pol);
-            tma_load_3d(kb + kHalfBytes, &kmap, 64, tt * kTile, unit, &ms->k_full[ks], pol);
+            const CUtensorMap *km = &lp.kmap[unit / p.upl];
+            const int local = unit % p.upl;
+            tma_load_3d(kb, km, 0, tt * kTile, local, &ms->k_full[ks], pol);
+            tma_load_3d(kb + kHalfBytes, km, 64, tt * kTile, local, &ms->k_full[ks], pol);
             ++kcount;
           }
         }
@@ -380,9 +392,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       warp_wait(&ms->q_empty[qs], ((k / kNQ) & 1) ^ 1, ms, p.status);
       tc_fence_after();
       const ItemRef it = item_of(p, k);
-      const int b = it.unit / p.Hkv, h = it.unit % p.Hkv;
+      const int layer = it.unit / p.upl, local = it.unit % p.upl;
+      const int b = local / p.Hkv, h = local % p.Hkv;
       const size_t row = (size_t)(b * p.Hq + h * p.G) * p.W + r;
-      const uint4 *src = reinterpret_cast<const uint4 *>(p.q + row * 256 + wg * 128);
+      const uint4 *src = reinterpret_cast<const uint4 *>(p.q[layer] + row * 256 + wg * 128);
       uint32_t w[32];
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
@@ -557,19 +570,21 @@ bool score_tc1_supported(const LayerGeom &g) {
   return g.dtype == RIPPLE_BF16 && g.D == 128 && g.R == 128 && g.P > 0 && encode_fn() != nullptr;
 }
 
-cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *k,
-                             const CompressWs &ws, float *votes, int32_t *status,
-                             cudaStream_t st) {
+cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const *q_win,
+                             const void *const *k, const CompressWs &ws, float *votes,
+                             int32_t *status, cudaStream_t st) {
   EncodeTiledFn enc = encode_fn();
-  if (enc == nullptr) return cudaErrorNotSupported;
-  CUtensorMap kmap;
-  {
+  if (enc == nullptr || n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorNotSupported;
+  static Tc1Launch lp;  // large: kept off the stack, filled under the lock
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int l = 0; l < n_layers; ++l) {
     cuuint64_t dims[3] = {128, (cuuint64_t)g.T, (cuuint64_t)g.units};
     cuuint64_t strides[2] = {256, (cuuint64_t)g.T * 256};
     cuuint32_t box[3] = {64, 128, 1};
     cuuint32_t es[3] = {1, 1, 1};
-    if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k), dims, strides, box,
-            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    if (enc(&lp.kmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k[l]), dims,
+            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
@@ -577,8 +592,9 @@ cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (sms <= 0) sms = 1;
-  Tc1Params p;
-  p.units = g.units;
+  Tc1Params &p = lp.p;
+  p.upl = g.units;
+  p.units = g.units * n_layers;
   p.T = g.T;
   p.P = g.P;
   p.W = g.W;
@@ -592,21 +608,21 @@ cudaError_t launch_score_tc1(const LayerGeom &g, const void *q_win, const void *
   const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
   p.tpi = tpi_min > kMinTilesPerItem ? tpi_min : kMinTilesPerItem;
   p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
-  p.total_items = g.units * p.n_ch;
+  p.total_items = p.units * p.n_ch;
   p.scale2 = g.scale2;
-  p.q = (const uint8_t *)q_win;
+  for (int l = 0; l < n_layers; ++l) p.q[l] = (const uint8_t *)q_win[l];
   p.partial = ws.row_partial;
   p.lognorm = ws.row_lognorm;
   p.votes = votes;
   p.ctrl = ws.counters;
   p.status = status;
-  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * g.units, st);
+  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * p.units, st);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(score_tc1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            kSmemBytes);
   if (e != cudaSuccess) return e;
   const int grid = p.total_items < sms ? p.total_items : sms;
-  void *args[] = {(void *)&kmap, (void *)&p};
+  void *args[] = {(void *)&lp};
   e = cudaLaunchCooperativeKernel((const void *)score_tc1_kernel, dim3(grid), dim3(kThreads), args,
                                   (size_t)kSmemBytes, st);
   count_launches(1);

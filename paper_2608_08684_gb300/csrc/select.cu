@@ -282,8 +282,16 @@ __device__ __forceinline__ int cta_exclusive_scan(int x, int *warp_tot, int *tot
   return res;
 }
 
+// Layers of one launch: units per layer, and per layer the kept count and the
+// index output [upl][n_keep].
+struct SelTable {
+  int upl;
+  int n_keep[kCompressMaxLayers];
+  int32_t *idx[kCompressMaxLayers];
+};
+
 __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
-    select_cluster_kernel(LayerGeom g, const float *votes, int n_keep, int32_t *idx) {
+    select_cluster_kernel(LayerGeom g, const float *votes, const __grid_constant__ SelTable tab) {
   extern __shared__ uint32_t sm[];
   uint32_t *hist2 = sm;                            // [2][kBins], one per round parity
   int *warp_tot = (int *)(sm + 2 * kBins);         // [33]
@@ -293,12 +301,14 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
   uint32_t *keys = sm + 2 * kBins + kCtrlWords;    // [S]
 
   const uint32_t rank = cluster_rank();
-  const int unit = blockIdx.x / kCluster;
+  const int unit = blockIdx.x / kCluster;  // over all layers of the launch
+  const int layer = unit / tab.upl;
+  const int n_keep = tab.n_keep[layer];
   const int P = g.P, K = n_keep - g.W;
   const int S = ((P + kCluster - 1) / kCluster + 31) & ~31;
   const int k0 = min(P, (int)rank * S), k1 = min(P, k0 + S);
   const float *v = votes + (size_t)unit * P;
-  int32_t *out = idx + (size_t)unit * n_keep;
+  int32_t *out = tab.idx[layer] + (size_t)(unit % tab.upl) * n_keep;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
 
   if (rank == 0)
@@ -483,27 +493,41 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
 
 }  // namespace
 
-cudaError_t launch_select(const LayerGeom &g, const float *votes, const CompressWs &ws,
-                          int n_keep, int32_t *idx, cudaStream_t st) {
+cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
+                          const CompressWs &ws, const int *n_keep, int32_t *const *idx,
+                          cudaStream_t st) {
+  if (n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorInvalidValue;
   const int per_cta = ((g.P + kCluster - 1) / kCluster + 31) & ~31;
-  if (per_cta <= kCMaxKeys && (long long)g.units * kCluster <= 0x7fffffff) {
+  if (per_cta <= kCMaxKeys && (long long)g.units * n_layers * kCluster <= 0x7fffffff) {
+    SelTable tab;
+    tab.upl = g.units;
+    for (int l = 0; l < n_layers; ++l) {
+      tab.n_keep[l] = n_keep[l];
+      tab.idx[l] = idx[l];
+    }
     // histograms, control words, keys, staged votes (with the pooling halo)
     const size_t smem = sizeof(uint32_t) * (2 * kBins + kCtrlWords + 2 * per_cta + 32);
     cudaError_t e = cudaFuncSetAttribute(select_cluster_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    select_cluster_kernel<<<g.units * kCluster, kCThreads, smem, st>>>(g, votes, n_keep, idx);
+    select_cluster_kernel<<<g.units * n_layers * kCluster, kCThreads, smem, st>>>(g, votes, tab);
     count_launches(1);
     return cudaGetLastError();
   }
+  // Very long prefixes: one CTA per unit, layer by layer.
   const int in_smem = g.P <= kSelectSmemKeys;
   const size_t smem = sizeof(uint32_t) * (kBins + kCtrlWords + (in_smem ? g.P : 0));
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  select_kernel<<<g.units, kThreads, smem, st>>>(g, votes, ws.keys, n_keep, in_smem, idx);
-  count_launches(1);
-  return cudaGetLastError();
+  for (int l = 0; l < n_layers; ++l) {
+    select_kernel<<<g.units, kThreads, smem, st>>>(g, votes + (size_t)l * g.units * g.P, ws.keys,
+                                                   n_keep[l], in_smem, idx[l]);
+    count_launches(1);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 __global__ void iota_kernel(int T, int32_t *idx) {

@@ -23,6 +23,7 @@ F32, BF16 = 0, 1
 POOL_MAX, POOL_AVG, POOL_NONE = 0, 1, 2
 OK, EINVAL, EWORKSPACE, EFULL, ECUDA, ETIMEOUT, EBOUNDS = range(7)
 MAX_LAYERS = 128
+COMPRESS_MAX_LAYERS = 80
 _POOLS = {"max": POOL_MAX, "avg": POOL_AVG, "none": POOL_NONE}
 _DTYPES = {torch.float32: F32, torch.bfloat16: BF16}
 
@@ -61,6 +62,15 @@ _lib.ripple_compress_workspace_bytes.restype = _i32
 _lib.ripple_compress_layer.argtypes = [ctypes.POINTER(LayerDesc), _i64, _p, _p, _p, _p, _p, _i32,
                                        _p, _p, ctypes.POINTER(_i32), _p, _sz, _p, _p]
 _lib.ripple_compress_layer.restype = _i32
+_lib.ripple_compress_layers_workspace_bytes.argtypes = [ctypes.POINTER(LayerDesc), _i32,
+                                                        ctypes.POINTER(_sz)]
+_lib.ripple_compress_layers_workspace_bytes.restype = _i32
+_lib.ripple_compress_layers.argtypes = [ctypes.POINTER(LayerDesc), _i32, ctypes.POINTER(_i64),
+                                        ctypes.POINTER(_p), ctypes.POINTER(_p), ctypes.POINTER(_p),
+                                        ctypes.POINTER(_p), ctypes.POINTER(_p),
+                                        ctypes.POINTER(_i32), ctypes.POINTER(_p),
+                                        ctypes.POINTER(_i32), _p, _sz, _p, _p]
+_lib.ripple_compress_layers.restype = _i32
 _lib.ripple_select_layer.argtypes = [ctypes.POINTER(LayerDesc), _i64, _p, _p, _p, _p, _p, _i32, _p,
                                      ctypes.POINTER(_i32), _p, _sz, _p, _p]
 _lib.ripple_select_layer.restype = _i32
@@ -159,6 +169,43 @@ def ripple_compress_layer(desc: LayerDesc, budget: int, q_win, k, v, k_out, v_ou
                                       _ptr(dev_status), _stream(stream)),
            "ripple_compress_layer")
     return n.value
+
+
+def ripple_compress_layers_workspace_bytes(desc: LayerDesc, n_layers: int) -> int:
+    out = _sz()
+    _check(_lib.ripple_compress_layers_workspace_bytes(ctypes.byref(desc), int(n_layers),
+                                                       ctypes.byref(out)),
+           "ripple_compress_layers_workspace_bytes")
+    return out.value
+
+
+class CompressTables:
+    """Host arrays of per-layer device pointers for ripple_compress_layers,
+    built once for a set of layer tensors (lists with one entry per layer)."""
+
+    def __init__(self, q_win, k, v, k_out, v_out, idx_out):
+        L = len(k)
+        self.n_layers = L
+        arr = lambda ts: (_p * L)(*[_ptr(x) for x in ts])
+        self.q, self.k, self.v = arr(q_win), arr(k), arr(v)
+        self.k_out, self.v_out, self.idx = arr(k_out), arr(v_out), arr(idx_out)
+        self.caps = (_i32 * L)(*[int(x.shape[-2]) for x in k_out])
+        self._keep = (list(q_win), list(k), list(v), list(k_out), list(v_out), list(idx_out))
+
+
+def ripple_compress_layers(desc: LayerDesc, budgets, tables: CompressTables, workspace,
+                           dev_status=None, stream=None) -> list:
+    """Compress tables.n_layers layers of one shape in one call; returns n_l per layer."""
+    L = tables.n_layers
+    b = (_i64 * L)(*[int(x) for x in budgets])
+    n = (_i32 * L)()
+    _check(_lib.ripple_compress_layers(ctypes.byref(desc), L, b, tables.q, tables.k, tables.v,
+                                       tables.k_out, tables.v_out, tables.caps, tables.idx, n,
+                                       _ptr(workspace),
+                                       workspace.numel() * workspace.element_size(),
+                                       _ptr(dev_status), _stream(stream)),
+           "ripple_compress_layers")
+    return [int(x) for x in n]
 
 
 def ripple_select_layer(desc: LayerDesc, budget: int, votes, k, v, k_out, v_out, idx_out,

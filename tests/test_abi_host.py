@@ -114,3 +114,18 @@ def test_entry_points_reject_before_any_cuda_work(lib):
                                 None, 0, None, None)
     assert st == lib.EINVAL
     assert lib.status_string(lib.EFULL) == "cache full"
+
+
+def test_compress_layers_host_validation(lib):
+    d = lib.layer_desc(4, 32, 8, 128, 32768, 32)
+    one = lib.ripple_compress_workspace_bytes(d)
+    four = lib.ripple_compress_layers_workspace_bytes(d, 4)
+    assert four >= 4 * 4 * 8 * 32736 * 4 and four > one
+    for bad in (0, -1, lib.COMPRESS_MAX_LAYERS + 1):
+        with pytest.raises(lib.RippleError):
+            lib.ripple_compress_layers_workspace_bytes(d, bad)
+    raw = ctypes.CDLL(lib.LIB_PATH)
+    n = (ctypes.c_int32 * 2)()
+    st = raw.ripple_compress_layers(ctypes.byref(d), 2, None, None, None, None, None, None,
+                                    None, None, n, None, 0, None, None)
+    assert st == lib.EINVAL

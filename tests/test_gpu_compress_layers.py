@@ -1,0 +1,71 @@
+"""ripple_compress_layers (several layers of one shape in one call, each with
+its own budget) gives, layer by layer, exactly what ripple_compress_layer
+gives: the same kept counts, indices and gathered rows, bit for bit. The
+single-layer path is checked against the oracle in test_gpu_compress.py."""
+import pytest
+import torch
+
+from paper_2608_08684_gb300 import synth
+from tests import gpu_common as C
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def _both(lib, wl, budgets, cap_extra=2, device_gen="cpu"):
+    L = len(budgets)
+    desc = lib.layer_desc(wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.seq_len,
+                          wl.window, wl.pool_kernel, "max", wl.torch_dtype)
+    B, H, d = wl.batch, wl.n_kv_heads, wl.head_dim
+    ins = [tuple(t.to(DEV) for t in C.layer_inputs(wl, l, device_gen)) for l in range(L)]
+    ns = [lib.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    k_out = [torch.zeros(B, H, n + cap_extra, d, dtype=wl.torch_dtype, device=DEV) for n in ns]
+    v_out = [torch.zeros_like(x) for x in k_out]
+    idx = [torch.full((B * H * max(n, 1),), -1, dtype=torch.int32, device=DEV) for n in ns]
+    tables = lib.CompressTables([x[0] for x in ins], [x[1] for x in ins], [x[2] for x in ins],
+                                k_out, v_out, idx)
+    ws = torch.empty(lib.ripple_compress_layers_workspace_bytes(desc, L), dtype=torch.uint8,
+                     device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    got = lib.ripple_compress_layers(desc, budgets, tables, ws, dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert got == ns
+    for l in range(L):
+        q, k, v = ins[l]
+        ref = C.run_compress(lib, wl, budgets[l], q, k, v, cap_extra=cap_extra, scores=False)
+        assert int(ref["status"].item()) == 0
+        n = ns[l]
+        assert torch.equal(idx[l][:B * H * n].view(B, H, n), ref["idx"]), f"layer {l} indices"
+        assert torch.equal(k_out[l], ref["k_out"]), f"layer {l} keys"
+        assert torch.equal(v_out[l], ref["v_out"]), f"layer {l} values"
+
+
+SHAPES = [
+    # tensor-core path (G * w = 128): all layers in three launches
+    ("bf16-d128-G4", dict(n_layers=6, batch=2, n_q_heads=8, n_kv_heads=2, head_dim=128,
+                          seq_len=1000, dtype="bf16", kv_dist="scaled_sinks", seed=21),
+     [0, 31, 32, 200, 968, 10**6]),
+    ("bf16-d128-G4-one-tile", dict(n_layers=3, batch=1, n_q_heads=4, n_kv_heads=1,
+                                   head_dim=128, seq_len=130, dtype="bf16", seed=22), [40, 98, 129]),
+    # other shapes: layer by layer inside the call
+    ("bf16-d128-G8", dict(n_layers=3, batch=1, n_q_heads=16, n_kv_heads=2, head_dim=128,
+                          seq_len=700, dtype="bf16", seed=23), [300, 50, 699]),
+    ("f32-d64-G2", dict(n_layers=4, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=64,
+                        seq_len=300, dtype="f32", seed=24), [64, 10, 300, 128]),
+]
+
+
+@pytest.mark.parametrize("name,over,budgets", SHAPES, ids=[s[0] for s in SHAPES])
+def test_layers_call_equals_per_layer_calls(lib, name, over, budgets):
+    wl = synth.WORKLOADS["tiny"].replace(**over)
+    _both(lib, wl, budgets)
+
+
+def test_layers_call_full_size_four_layers(lib):
+    # four layers of the 32k workload with its allocator budgets, inputs on the GPU
+    wl = synth.WORKLOADS["llama8b-32k"]
+    b = lib.ripple_alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
+                                 wl.global_budget)
+    wl4 = wl.replace(n_layers=4)
+    _both(lib, wl4, [b[12], b[0], b[20], b[31]], device_gen=DEV)
