@@ -191,6 +191,8 @@ ripple_status ripple_compress_layers_workspace_bytes(const ripple_layer_desc *de
  *              256-byte aligned, no initialisation needed
  * Errors: RIPPLE_EINVAL (as ripple_compress_layer, for any layer),
  * RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status as ripple_compress_layer.
+ * The call may be captured in a CUDA graph (no host synchronisation, no
+ * allocation).
  */
 ripple_status ripple_compress_layers(const ripple_layer_desc *desc, int32_t n_layers,
                                      const int64_t *budgets_host, const void *const *q_win_host,
@@ -267,6 +269,8 @@ ripple_status ripple_decode_workspace_bytes(const ripple_decode_desc *desc,
  * Consecutive calls on one stream may overlap: a call's thread blocks may
  * start while the previous call's last blocks finish; they read nothing the
  * previous call writes before it has completed.
+ * The call may be captured in a CUDA graph (no host synchronisation, no
+ * allocation); capture was tested after one call outside the capture.
  * A layer with lens[l] >= caps_host[l] (or lens[l] < 0) is not appended to,
  * its output rows are zero, its length is unchanged, and RIPPLE_EFULL is
  * written to *dev_status.
