@@ -428,16 +428,16 @@ def run_ours(args, rank, world, local_rank):
     dec_gbs = st.decode_bytes_per_step() / (dec_avg / 1e3) / 1e9
     comp_total = comp_avg
     dec_total = dec_avg * wl.decode_steps
-    dec_traffic = profile_traffic("decode_tc_kernel_llama3-8b_B4_T32768.md",
-                                  ["decode_tc.cu", "decode.cuh", "tc_ptx.cuh", "common.cuh"],
+    dec_traffic = profile_traffic("decode_kernel_llama3-8b_B4_T32768.md",
+                                  ["decode.cu", "decode.cuh", "common.cuh"],
                                   st.decode_bytes_per_step()) \
         if wl.name.startswith("llama3-8b-32L-32q8kv-d128-B4-T32768") else None
     roof_dec = {"bound": "hbm", "achieved": round(dec_gbs, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(dec_gbs / hbm, 4), "traffic": dec_traffic,
                 "traffic_source": ("ncu dram bytes of the first decode step "
-                                   "(profiles/decode_tc_kernel_llama3-8b_B4_T32768.md), scaled "
+                                   "(profiles/decode_kernel_llama3-8b_B4_T32768.md), scaled "
                                    "by algorithmic bytes") if dec_traffic else None,
-                "kernel": "decode_tc_kernel (ripple_decode_attn, one launch per step)",
+                "kernel": "decode_kernel (ripple_decode_attn, one launch per step)",
                 "bytes_per_launch": round(st.decode_bytes_per_step()),
                 "ms_per_launch": round(dec_avg, 5), "peak_source": hbm_src}
     comp_traffic = profile_traffic("compress_kernels_llama3-8b_B4_T32768_layer12.md",

@@ -258,11 +258,10 @@ ripple_status ripple_decode_workspace_bytes(const ripple_decode_desc *desc,
  *              read, then incremented by one per layer
  * out          device fp32 [L][B][Hq][d]
  * workspace    device scratch of at least ripple_decode_workspace_bytes bytes.
- *              Its leading block holds the step's work counters. For bf16,
- *              d = 128 and at most 80 layers (the tensor-core path) every call
+ *              Its leading block holds the step's work counters. Every call
  *              leaves that block at zero, and the library clears it only when
- *              the workspace differs from the one its previous such call on
- *              the device used; so between consecutive calls with the same
+ *              the workspace differs from the one its previous call on the
+ *              device used; so between consecutive calls with the same
  *              workspace the caller must not write into it (another buffer
  *              is fine). After a call that ended with RIPPLE_ETIMEOUT in
  *              *dev_status, pass a different workspace or zero the block.
@@ -307,8 +306,7 @@ ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
  *   caps) > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
  * - Every call on a device shares the one array. Its counters start at zero
  *   (the array is zero-initialised when the library is loaded) and every call
- *   leaves them at zero (the tensor-core path resets them as it exits; other
- *   paths clear them with a memset enqueued on `stream` first); every partial
+ *   leaves them at zero (the kernel resets them as it exits); every partial
  *   a call reads it has rewritten, so nothing carries over from the previous
  *   call. A call that ended with RIPPLE_ETIMEOUT may leave the counters
  *   dirty: later calls of this entry point on that device are then invalid.

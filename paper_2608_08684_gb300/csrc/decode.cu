@@ -1,26 +1,42 @@
 // GQA decode attention over the ragged compressed caches (Sec. 4.1: each new
 // query attends to the cached states), with the append of the new token.
 //
-// One persistent launch per step covers every layer; one CTA per SM with 16
-// compute warps and one producer warp. Work item = up to kItemSub sub-chunks
-// of one (layer, batch row, KV head) group's cache rows; items are fetched
-// with an atomic counter, layers with the longest caches first (longest-
-// processing-time order). The producer warp stages each sub-chunk's K and V
-// rows in shared memory with bulk-async (TMA engine) copies, two stages
-// deep plus an L2 prefetch further ahead, and writes the new token's rows into
-// the stage (and appends them to the cache). Every compute warp owns CR/16
-// rows of each sub-chunk and keeps its
-// own online-softmax state, so no block-wide barrier is needed per sub-chunk
-// (stages are released through mbarriers):
-//   scores  q_g . k_row * scale * log2(e): S lanes per row, the query slice in
-//           registers, packed fp32x2 FMAs, a reduce-scatter over the S lanes
-//           that leaves each lane with one head's full dot product;
-//   softmax per head over the warp's rows (running max / sum per warp);
-//   output  lanes over head dims, probabilities broadcast from shared memory.
-// At an item's end the 16 warps' states are merged; an item covering its
-// whole group writes the output, otherwise its unnormalised partial is stored
-// and the group's last finishing item (atomic count) combines the partials in
-// item order (deterministic). The last CTA to exit advances the lengths.
+// One persistent launch per step covers every layer; one CTA per SM with 8
+// compute warps and one producer warp. Work item = up to kItemRows cache rows
+// of one (layer, batch row, KV head) group; items are fetched with an atomic
+// counter (one ahead), layers with the longest caches first. The producer
+// stages each item's G query rows and then its sub-chunks of K and V rows in
+// shared memory with bulk-async copies (TMA engine) through a ring of stages;
+// the new token's key and value rows are copied into the stage behind the
+// cached rows, and appended to the cache from there.
+//
+// Lane layout (the same for Q.K and P.V): the rows of a warp step are split
+// over R row groups of S lanes; each lane owns DL head dims (its 16-byte
+// pieces of the row) of every query head of the group: it reads those dims of
+// the scaled fp32 queries from shared memory (converted once per item, in the
+// order the lanes read them) and keeps those dims of the output accumulator
+// in registers. Per row:
+//   scores   fp32x2 FMAs over the lane's dims, then a reduce-scatter over the
+//            S lanes of the row group (warp shuffles) that leaves each lane
+//            with the full dot product of one head;
+//   softmax  each (row group, head) keeps its own running max and sum (online
+//            softmax; the max is moved, and the state rescaled, only when a
+//            score exceeds it by more than 2^8, so rescaling is rare);
+//            the probability is computed once per head and all-gathered over
+//            the row group (warp shuffles);
+//   output   fp32x2 FMAs of the probabilities with the lane's value dims.
+// At an item's end the row groups of a warp are merged by a shuffle butterfly
+// and the 8 warps through shared memory. An item covering its whole group
+// writes the output; otherwise its unnormalised partial is stored and the
+// group's last finishing item (atomic count) combines the partials in item
+// order (deterministic).
+//
+// Counters are left at zero by the kernel itself (the group combiner and the
+// last CTA to leave reset them), and each launch is a programmatic dependent
+// of the previous one on the stream: its CTAs take SMs as the previous step's
+// CTAs leave and wait (griddepcontrol.wait) until that step has completed.
+// Every wait is bounded; on timeout the CTA raises RIPPLE_ETIMEOUT and all
+// roles leave their loops together.
 #include <math.h>
 
 #include <mutex>
@@ -32,50 +48,67 @@
 namespace ripple {
 namespace {
 
-constexpr int kWarps = 16;                    // compute warps
+constexpr int kWarps = 8;                     // compute warps
 constexpr int kThreads = (kWarps + 1) * 32;   // + one producer warp
-constexpr int kStageBytes = 32768;            // K (or V) bytes of one sub-chunk
-constexpr int kStages = 2;
-constexpr int kItemSub = 16;                  // sub-chunks per work item (merges are costly)
+constexpr int kMaxStageBytes = 32768;         // K (or V) bytes of one sub-chunk, at most
+constexpr int kRowsPerGroup = 4;              // rows per row group and sub-chunk (warp steps)
 constexpr int kItemSlots = 4;
-constexpr int kPrefetchAhead = 2;             // sub-chunks prefetched into L2 past the stages
+constexpr int kMaxStages = 6;
+// Lazy rescaling: a running max is only moved when a score exceeds it by more
+// than 2^kRescaleLog2 (probabilities relative to a stale max stay <= 2^8).
+constexpr float kRescaleLog2 = 8.f;
+constexpr int kSmemBudget = 226 * 1024;
+constexpr int kMiscBytes = 4096;              // barriers, work list, merge statistics
+constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at the SM clock
+constexpr unsigned kFull = 0xffffffffu;
+
+constexpr int cmax(int a, int b) { return a > b ? a : b; }
+constexpr int cmin(int a, int b) { return a < b ? a : b; }
 
 template <typename Tin, int D, int G>
 struct DecCfg {
   static constexpr int ROW_BYTES = D * (int)sizeof(Tin);
-  static constexpr int CR = kStageBytes / ROW_BYTES;     // rows per sub-chunk
-  static constexpr int ITEM_ROWS = CR * kItemSub;
-  static constexpr int RPW = CR / kWarps;                // rows per warp per sub-chunk
-  static constexpr int S = G <= 2 ? 8 : (G == 4 ? 16 : 32);  // lanes per row in the scores
-  static constexpr int PB0 = ROW_BYTES / S;
-  static constexpr int PB = PB0 < 16 ? PB0 : 16;         // bytes per piece
-  static constexpr int PIECES = ROW_BYTES / PB;          // pieces per row
-  static constexpr int PE = PB / (int)sizeof(Tin);       // elements per piece
-  static constexpr int PPL = PIECES / S;                 // pieces per lane
-  static constexpr int NPIECE = ROW_BYTES / 16;          // 16-byte units per row
-  static constexpr int DL = PPL * PE;                    // dims per lane in the scores
-  static constexpr int RPI = 32 / S;                     // rows per warp step
-  static constexpr int NIT = RPW / RPI;                  // warp steps per sub-chunk
-  static constexpr int HL = S / G;                       // lanes per head after reduce-scatter
-  static constexpr int DV = D / 32;                      // dims per lane in the output
-  static_assert(NIT >= 1 && RPW % RPI == 0, "rows per warp");
-  static_assert(PPL * S == PIECES && HL >= 1, "lanes per row");
-  static_assert(DL % 2 == 0 && DV % 2 == 0, "fp32x2 pairs");
+  static constexpr int NPIECE = ROW_BYTES / 16;             // 16-byte pieces per row
+  static constexpr int PE = 16 / (int)sizeof(Tin);          // elements per piece
+  // lanes per row: the queries and accumulators of a lane stay at 64
+  // registers each, at least one lane per head, and a warp step's rows fit a
+  // sub-chunk
+  static constexpr int S = cmax(cmax(G * D / 64, G), cmax(ROW_BYTES / 128, 1));
+  static constexpr int R = 32 / S;                          // row groups (rows per warp step)
+  static constexpr int NIT =                                // warp steps per sub-chunk
+      cmax(1, cmin(kRowsPerGroup, kMaxStageBytes / (kWarps * R * ROW_BYTES)));
+  static constexpr int RPW = R * NIT;                       // rows per warp per sub-chunk
+  static constexpr int CR = RPW * kWarps;                   // rows per sub-chunk
+  static constexpr int STAGE_BYTES = CR * ROW_BYTES;
+  static constexpr int PPL = NPIECE / S;                    // pieces per lane
+  static constexpr int DL = PPL * PE;                       // head dims per lane
+  static constexpr int HL = S / G;                          // lanes per head after the reduce-scatter
+  static constexpr int QBYTES = G * ROW_BYTES;              // one group's queries
+  static constexpr int NH = PE / 4;                         // float4 per piece in fp32
+  static constexpr int STAGES =
+      cmin(kMaxStages, (kSmemBudget - kMiscBytes - kItemSlots * QBYTES - (kWarps + 2) * G * D * 4) /
+                           (2 * STAGE_BYTES));
+  static_assert(kItemRows % CR == 0, "items are whole sub-chunks");
+  static_assert(S <= 32 && S <= NPIECE && NPIECE % S == 0, "lanes per row");
+  static_assert(STAGE_BYTES <= kMaxStageBytes, "stage size");
+  static_assert(DL % 2 == 0 && PE % 2 == 0, "fp32x2 pairs");
+  static_assert(STAGES >= 2, "shared memory budget");
 };
 
 template <typename Tin, int D, int G>
 struct DecSmem {
   using C = DecCfg<Tin, D, G>;
-  alignas(128) uint8_t kv[kStages][2][kStageBytes];  // [stage][K, V]
-  alignas(16) float red_o[kWarps][G * D];             // per-warp outputs at an item's end
-  alignas(16) float pw[kWarps][C::RPW][G];            // per-warp probabilities
-  alignas(16) float aw[kWarps][G];                    // per-warp rescale factors
+  alignas(128) uint8_t kv[C::STAGES][2][C::STAGE_BYTES];  // [stage][K, V]
+  alignas(128) uint8_t qs[kItemSlots][C::QBYTES];      // each item's query rows
+  alignas(16) float qf[2][G * D];                      // scaled fp32 queries, lane-piece order
+  alignas(16) float red_o[kWarps][G * D];              // per-warp outputs at an item's end
   float red_m[kWarps][G], red_l[kWarps][G];
-  uint64_t full[kStages], empty[kStages], item_full[kItemSlots], item_empty[kItemSlots];
+  uint64_t full[C::STAGES], empty[C::STAGES], item_full[kItemSlots], item_empty[kItemSlots];
   int item_id[kItemSlots];
   int len[RIPPLE_MAX_LAYERS];    // by work-order position; -1 = full layer
   int nch[RIPPLE_MAX_LAYERS];    // items per group, by work-order position
   int base[RIPPLE_MAX_LAYERS + 1];
+  int abort_flag;
   int last;
 };
 
@@ -83,10 +116,8 @@ struct ItemInfo {
   int pos, layer, group, b, h, chunk, nch, len, r0, rows, full;
 };
 
-template <typename Tin, int D, int G>
-__device__ __forceinline__ ItemInfo item_info(const DecParams &p, const DecSmem<Tin, D, G> &s,
-                                              int it) {
-  using C = DecCfg<Tin, D, G>;
+template <typename S>
+__device__ __forceinline__ ItemInfo item_info(const DecParams &p, const S &s, int it) {
   int lo = 0, hi = p.L - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
@@ -104,9 +135,43 @@ __device__ __forceinline__ ItemInfo item_info(const DecParams &p, const DecSmem<
   f.group = (f.layer * p.B + f.b) * p.Hkv + f.h;
   f.len = s.len[lo];
   f.full = f.len < 0;
-  f.r0 = f.chunk * C::ITEM_ROWS;
-  f.rows = f.full ? 0 : min(C::ITEM_ROWS, f.len + 1 - f.r0);
+  f.r0 = f.chunk * kItemRows;
+  // rows 0..len: the cached rows and the new token
+  f.rows = f.full ? 0 : min(kItemRows, f.len + 1 - f.r0);
   return f;
+}
+
+// Bounded wait on an mbarrier phase. Gives up when another role of the CTA
+// has given up, or after ~kWaitCycles (then raises the CTA's abort flag and
+// reports RIPPLE_ETIMEOUT).
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, int *abort_flag,
+                                         int32_t *status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*(volatile int *)abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *(volatile int *)abort_flag = 1;
+      report(status, RIPPLE_ETIMEOUT);
+      return false;
+    }
+  }
+}
+
+// Named barrier over the compute warps that also ORs a predicate over them.
+__device__ __forceinline__ bool compute_bar_or(bool pred) {
+  __syncwarp();
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n"
+      " setp.ne.u32 p, %1, 0;\n"
+      " barrier.red.or.pred q, 1, %2, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "n"(kWarps * 32)
+      : "memory");
+  return r != 0;
 }
 
 // 2*NP consecutive elements (one aligned load of 4 * NP bytes for bf16, or
@@ -117,66 +182,367 @@ __device__ __forceinline__ float2 bf16x2_pair(uint32_t w) {
 }
 template <int NP>
 __device__ __forceinline__ void load_pairs(const __nv_bfloat16 *p, float2 (&o)[NP]) {
-  if constexpr (NP == 4) {
-    const uint4 u = *reinterpret_cast<const uint4 *>(p);
-    o[0] = bf16x2_pair(u.x); o[1] = bf16x2_pair(u.y);
-    o[2] = bf16x2_pair(u.z); o[3] = bf16x2_pair(u.w);
-  } else if constexpr (NP == 2) {
-    const uint2 u = *reinterpret_cast<const uint2 *>(p);
-    o[0] = bf16x2_pair(u.x); o[1] = bf16x2_pair(u.y);
-  } else {
-    static_assert(NP == 1, "pairs");
-    o[0] = bf16x2_pair(*reinterpret_cast<const uint32_t *>(p));
-  }
+  static_assert(NP == 4, "one 16-byte piece");
+  const uint4 u = *reinterpret_cast<const uint4 *>(p);
+  o[0] = bf16x2_pair(u.x); o[1] = bf16x2_pair(u.y);
+  o[2] = bf16x2_pair(u.z); o[3] = bf16x2_pair(u.w);
 }
 template <int NP>
 __device__ __forceinline__ void load_pairs(const float *p, float2 (&o)[NP]) {
-  if constexpr (NP == 2) {
-    const float4 u = *reinterpret_cast<const float4 *>(p);
-    o[0] = make_float2(u.x, u.y);
-    o[1] = make_float2(u.z, u.w);
-  } else {
-    static_assert(NP == 1, "pairs");
-    o[0] = *reinterpret_cast<const float2 *>(p);
-  }
+  static_assert(NP == 2, "one 16-byte piece");
+  const float4 u = *reinterpret_cast<const float4 *>(p);
+  o[0] = make_float2(u.x, u.y);
+  o[1] = make_float2(u.z, u.w);
 }
 
-// L2 prefetch of one sub-chunk's cache rows (K and V, rows before the new
-// token); `sub` may run past the item's end into the following item.
-template <typename Tin, int D, int G>
-__device__ __forceinline__ void prefetch_sub(const DecParams &p, const DecSmem<Tin, D, G> &s,
-                                             int total, int it, int nxt, int sub) {
-  using C = DecCfg<Tin, D, G>;
-  if (it >= total) return;
-  ItemInfo f = item_info(p, s, it);
-  int nsub = f.full ? 0 : (f.rows + C::CR - 1) / C::CR;
-  if (sub >= nsub) {
-    sub -= nsub;
-    if (nxt >= total) return;
-    f = item_info(p, s, nxt);
-    nsub = f.full ? 0 : (f.rows + C::CR - 1) / C::CR;
-    if (sub >= nsub) return;
-  }
-  const int rs = f.r0 + sub * C::CR;
-  const int re = min(rs + C::CR, f.len);
-  if (re <= rs) return;
-  const size_t off = ((size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer] + rs) * C::ROW_BYTES;
-  const uint32_t bytes = (uint32_t)(re - rs) * C::ROW_BYTES;
-  bulk_prefetch_l2((const uint8_t *)p.kc[f.layer] + off, bytes);
-  bulk_prefetch_l2((const uint8_t *)p.vc[f.layer] + off, bytes);
-}
-
-template <int G>
-__device__ __forceinline__ void load_probs(const float *src, float (&pr)[G]) {
-  if constexpr (G % 4 == 0) {
+// Per-head values of a lane are kept in an order permuted by the lane's own
+// head hq = (lane % S) / (S / G): entry j holds head j ^ hq. Then every step
+// of the reduce-scatter and of the all-gather over the S lanes of a row group
+// is a plain shuffle (the partner's entry that this lane needs sits at a fixed
+// index), with no per-lane selects.
+//
+// Reduce-scatter of G per-lane partial sums: afterwards v[0] of every lane is
+// the full sum of its head hq. At the step over lane bit o the partner's head
+// differs from this lane's in the head bit being split, which is bit
+// log2(nv / 2) of the entry index.
+template <int S, int G>
+__device__ __forceinline__ void reduce_scatter(float (&v)[G]) {
 #pragma unroll
-    for (int i = 0; i < G; i += 4) {
-      const float4 x = *reinterpret_cast<const float4 *>(src + i);
-      pr[i] = x.x; pr[i + 1] = x.y; pr[i + 2] = x.z; pr[i + 3] = x.w;
+  for (int o = S / 2, nv = G; o >= 1; o >>= 1) {
+    if (nv > 1) {
+#pragma unroll
+      for (int i = 0; i < G / 2; ++i)
+        if (i < nv / 2) v[i] += __shfl_xor_sync(kFull, v[i + nv / 2], o);
+      nv /= 2;
+    } else {
+      v[0] += __shfl_xor_sync(kFull, v[0], o);
     }
-  } else {
+  }
+}
+
+// Inverse of the head split of reduce_scatter: from x (the value of head hq)
+// every lane of the row group receives o[j] = the value of head j ^ hq.
+template <int S, int G>
+__device__ __forceinline__ void all_gather(float x, float (&o)[G]) {
+  o[0] = x;
 #pragma unroll
-    for (int i = 0; i < G; ++i) pr[i] = src[i];
+  for (int lev = 0; (1 << lev) < G; ++lev)
+#pragma unroll
+    for (int i = 0; i < (1 << lev); ++i)
+      o[(1 << lev) + i] = __shfl_xor_sync(kFull, o[i], (S / G) << lev);
+}
+
+// ------------------------------------------------------------ producer
+template <typename Tin, int D, int G>
+__device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &s, int total) {
+  using C = DecCfg<Tin, D, G>;
+  const int units = p.B * p.Hkv;
+  uint32_t j = 0;
+  int it = atomicAdd(&p.ctrl[0], 1);
+  for (int icount = 0;; ++icount) {
+    const int slot = icount % kItemSlots;
+    const int nxt = it < total ? atomicAdd(&p.ctrl[0], 1) : total;
+    if (!wait_bar(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, &s.abort_flag, p.status))
+      return;
+    const int cur = min(it, total);
+    s.item_id[slot] = cur;
+    if (cur >= total) {
+      mbar_arrive(&s.item_full[slot]);
+      return;
+    }
+    const ItemInfo f = item_info(p, s, cur);
+    if (f.full) {
+      mbar_arrive(&s.item_full[slot]);
+    } else {
+      const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
+      mbar_arrive_expect_tx(&s.item_full[slot], C::QBYTES);
+      bulk_g2s(s.qs[slot], (const uint8_t *)p.q + qrow * C::ROW_BYTES, C::QBYTES,
+               &s.item_full[slot]);
+      const int nsub = (f.rows + C::CR - 1) / C::CR;
+      const size_t gbase = (size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer];
+      const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * C::ROW_BYTES;
+      for (int sub = 0; sub < nsub; ++sub, ++j) {
+        const int stage = j % C::STAGES;
+        if (!wait_bar(&s.empty[stage], ((j / C::STAGES) & 1) ^ 1, &s.abort_flag, p.status))
+          return;
+        const int rs = f.r0 + sub * C::CR;
+        const int re = min(rs + C::CR, f.len);  // rows >= len are not in the cache yet
+        const int nk = re > rs ? re - rs : 0;
+        const bool has_new = f.len >= rs && f.len < rs + C::CR;
+        mbar_arrive_expect_tx(&s.full[stage], 2u * (nk + (has_new ? 1 : 0)) * C::ROW_BYTES);
+        if (nk > 0) {
+          const size_t off = (gbase + rs) * C::ROW_BYTES;
+          bulk_g2s(s.kv[stage][0], (const uint8_t *)p.kc[f.layer] + off, nk * C::ROW_BYTES,
+                   &s.full[stage]);
+          bulk_g2s(s.kv[stage][1], (const uint8_t *)p.vc[f.layer] + off, nk * C::ROW_BYTES,
+                   &s.full[stage]);
+        }
+        if (has_new) {
+          const int r = f.len - rs;
+          bulk_g2s(s.kv[stage][0] + r * C::ROW_BYTES, (const uint8_t *)p.k_new + nb,
+                   C::ROW_BYTES, &s.full[stage]);
+          bulk_g2s(s.kv[stage][1] + r * C::ROW_BYTES, (const uint8_t *)p.v_new + nb,
+                   C::ROW_BYTES, &s.full[stage]);
+        }
+      }
+    }
+    it = nxt;
+  }
+}
+
+// ------------------------------------------------------------ compute warps
+template <typename Tin, int D, int G>
+__device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &s, int total,
+                                        int warp, int lane) {
+  using C = DecCfg<Tin, D, G>;
+  constexpr int S = C::S, R = C::R, NIT = C::NIT, PPL = C::PPL, PE = C::PE, DL = C::DL;
+  const int tid = warp * 32 + lane;
+  const int sl = lane % S;              // lane within its row group
+  const int rg = lane / S;              // row group
+  const int hq = sl / C::HL;            // head of this lane after the reduce-scatter;
+                                        // per-head arrays hold head j ^ hq at entry j
+  const int rw0 = warp * C::RPW;        // this warp's first row in a sub-chunk
+  uint32_t j = 0;
+  for (int icount = 0;; ++icount) {
+    const int slot = icount % kItemSlots;
+    bool ok = wait_bar(&s.item_full[slot], (icount / kItemSlots) & 1, &s.abort_flag, p.status);
+    ok = __all_sync(kFull, ok);
+    const int it = ok ? s.item_id[slot] : total;
+    // Queries to fp32, scaled to log2 units, in the order the lanes read them:
+    // [entry j][piece k][half h][lane sl][4], entry j of lane sl being head
+    // j ^ hq(sl).
+    float *qf = s.qf[icount & 1];
+    if (it < total) {
+      const Tin *qg = (const Tin *)s.qs[slot];
+      for (int e = tid; e < G * D; e += kWarps * 32) {
+        const int c = e % 4, l4 = (e / 4) % S, h = (e / (4 * S)) % C::NH;
+        const int k = (e / (4 * S * C::NH)) % PPL, jj = e / (4 * S * C::NH * PPL);
+        const int g = jj ^ (l4 / C::HL);
+        qf[e] = to_f32(qg[g * D + (l4 + k * S) * PE + h * 4 + c]) * p.scale2;
+      }
+    }
+    // All compute warps leave together (the item's merge has named barriers);
+    // this barrier also frees the merge buffers of the previous item and
+    // publishes the fp32 queries.
+    if (compute_bar_or(it >= total || *(volatile int *)&s.abort_flag)) {
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
+      break;
+    }
+    const ItemInfo f = item_info(p, s, it);
+    const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
+    if (f.full) {
+      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
+      for (int e = tid; e < G * D; e += kWarps * 32) p.out[qrow * D + e] = 0.f;
+      continue;
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&s.item_empty[slot]);
+
+    float2 acc[G][DL / 2];  // entry j: head j ^ hq, the lane's dims
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+#pragma unroll
+      for (int e = 0; e < DL / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
+    float m_run = -INFINITY, l_run = 0.f;  // of head hq over this row group's rows
+
+    // One sub-chunk of this warp's rows; kMask: some rows are past nrows
+    // (their index is clamped to a valid row and their probability is 0).
+    auto rows_step = [&](const Tin *ks, const Tin *vs, int nrows, auto mask_tag) {
+      constexpr bool kMask = decltype(mask_tag)::value;
+      float2 d2[NIT][G];
+#pragma unroll
+      for (int t = 0; t < NIT; ++t)
+#pragma unroll
+        for (int g = 0; g < G; ++g) d2[t][g] = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int k = 0; k < PPL; ++k) {
+        float2 kp[NIT][PE / 2];
+#pragma unroll
+        for (int t = 0; t < NIT; ++t) {
+          const int row = rw0 + t * R + rg;
+          const int rr = kMask ? min(row, nrows - 1) : row;
+          load_pairs<PE / 2>(ks + (size_t)rr * D + (sl + k * S) * PE, kp[t]);
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          float2 qp[PE / 2];
+#pragma unroll
+          for (int h = 0; h < C::NH; ++h) {
+            const float4 x =
+                *reinterpret_cast<const float4 *>(&qf[(((g * PPL + k) * C::NH + h) * S + sl) * 4]);
+            qp[2 * h] = make_float2(x.x, x.y);
+            qp[2 * h + 1] = make_float2(x.z, x.w);
+          }
+#pragma unroll
+          for (int t = 0; t < NIT; ++t)
+#pragma unroll
+            for (int e = 0; e < PE / 2; ++e) d2[t][g] = __ffma2_rn(qp[e], kp[t][e], d2[t][g]);
+        }
+      }
+      float sc[NIT];
+#pragma unroll
+      for (int t = 0; t < NIT; ++t) {
+        const int row = rw0 + t * R + rg;
+        float v[G];
+#pragma unroll
+        for (int g = 0; g < G; ++g) v[g] = d2[t][g].x + d2[t][g].y;
+        reduce_scatter<S, G>(v);
+        sc[t] = (!kMask || row < nrows) ? v[0] : -INFINITY;
+      }
+      float mb = sc[0];
+#pragma unroll
+      for (int t = 1; t < NIT; ++t) mb = fmaxf(mb, sc[t]);
+      const bool grow = mb > m_run + kRescaleLog2;  // true for the first rows (m_run = -inf)
+      if (__any_sync(kFull, grow)) {
+        const float mn = grow ? mb : m_run;
+        const float a = grow ? fast_exp2(m_run - mn) : 1.f;
+        l_run *= a;
+        float ag[G];
+        all_gather<S, G>(a, ag);
+#pragma unroll
+        for (int g = 0; g < G; ++g)
+#pragma unroll
+          for (int e = 0; e < DL / 2; ++e) acc[g][e] = __fmul2_rn(acc[g][e], make_float2(ag[g], ag[g]));
+        m_run = mn;
+      }
+#pragma unroll
+      for (int t = 0; t < NIT; ++t) {
+        const int row = rw0 + t * R + rg;
+        const int rr = kMask ? min(row, nrows - 1) : row;
+        const float pt =
+            (!kMask || sc[t] > -INFINITY) ? fast_exp2(sc[t] - m_run) : 0.f;  // m_run is finite
+        l_run += pt;
+        float pg[G];
+        all_gather<S, G>(pt, pg);
+#pragma unroll
+        for (int k = 0; k < PPL; ++k) {
+          float2 vp[PE / 2];
+          load_pairs<PE / 2>(vs + (size_t)rr * D + (sl + k * S) * PE, vp);
+#pragma unroll
+          for (int g = 0; g < G; ++g)
+#pragma unroll
+            for (int e = 0; e < PE / 2; ++e)
+              acc[g][k * PE / 2 + e] =
+                  __ffma2_rn(make_float2(pg[g], pg[g]), vp[e], acc[g][k * PE / 2 + e]);
+        }
+      }
+    };
+
+    const int nsub = (f.rows + C::CR - 1) / C::CR;
+    for (int sub = 0; sub < nsub; ++sub, ++j) {
+      const int stage = j % C::STAGES;
+      wait_bar(&s.full[stage], (j / C::STAGES) & 1, &s.abort_flag, p.status);
+      __syncwarp();
+      const int nrows = min(C::CR, f.rows - sub * C::CR);
+      const Tin *ks = (const Tin *)s.kv[stage][0];
+      const Tin *vs = (const Tin *)s.kv[stage][1];
+      if (rw0 + C::RPW <= nrows)
+        rows_step(ks, vs, nrows, std::false_type{});
+      else if (rw0 < nrows)
+        rows_step(ks, vs, nrows, std::true_type{});
+      // The new token's rows, staged behind the cached rows, go to the cache.
+      const int rs = f.r0 + sub * C::CR;
+      if (warp == 0 && f.len >= rs && f.len < rs + C::CR) {
+        const size_t dst = ((size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer] + f.len) * C::ROW_BYTES;
+        for (int e = lane; e < 2 * C::NPIECE; e += 32) {
+          const int kvsel = e >= C::NPIECE, pc = e % C::NPIECE;
+          const uint4 val = reinterpret_cast<const uint4 *>(
+              s.kv[stage][kvsel] + (size_t)(f.len - rs) * C::ROW_BYTES)[pc];
+          reinterpret_cast<uint4 *>((uint8_t *)(kvsel ? p.vc[f.layer] : p.kc[f.layer]) + dst)[pc] =
+              val;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.empty[stage]);
+    }
+
+    // Item end. (1) Merge the warp's row groups (butterfly over lanes with
+    // the same position in their row group, hence the same head).
+#pragma unroll
+    for (int o = S; o < 32; o <<= 1) {
+      const float mo = __shfl_xor_sync(kFull, m_run, o);
+      const float lo = __shfl_xor_sync(kFull, l_run, o);
+      const float M = fmaxf(m_run, mo);
+      const float as = m_run == -INFINITY ? 0.f : fast_exp2(m_run - M);
+      const float ao = mo == -INFINITY ? 0.f : fast_exp2(mo - M);
+      l_run = l_run * as + lo * ao;
+      m_run = M;
+      float gs[G], go[G];
+      all_gather<S, G>(as, gs);
+      all_gather<S, G>(ao, go);
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int e = 0; e < DL / 2; ++e) {
+          float2 other;
+          other.x = __shfl_xor_sync(kFull, acc[g][e].x, o);
+          other.y = __shfl_xor_sync(kFull, acc[g][e].y, o);
+          acc[g][e] = __ffma2_rn(acc[g][e], make_float2(gs[g], gs[g]),
+                                 __fmul2_rn(other, make_float2(go[g], go[g])));
+        }
+    }
+    // (2) Merge the 8 warps through shared memory.
+    if (rg == 0) {
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int k = 0; k < PPL; ++k)
+#pragma unroll
+          for (int e = 0; e < PE / 2; ++e)
+            *reinterpret_cast<float2 *>(
+                &s.red_o[warp][(g ^ hq) * D + (sl + k * S) * PE + 2 * e]) = acc[g][k * PE / 2 + e];
+      if (sl % C::HL == 0) {
+        s.red_m[warp][hq] = m_run;
+        s.red_l[warp][hq] = l_run;
+      }
+    }
+    named_bar_sync(1, kWarps * 32);
+    const bool single = f.nch == 1;
+    const int item_base = s.base[f.pos] + (f.b * p.Hkv + f.h) * f.nch;
+    const int item = item_base + f.chunk;
+    for (int e = tid; e < G * D; e += kWarps * 32) {
+      const int g = e / D;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, s.red_m[w][g]);
+      float num = 0.f, den = 0.f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        const float wgt = fast_exp2(s.red_m[w][g] - M);  // M is finite: row 0 is in warp 0
+        num += wgt * s.red_o[w][e];
+        den += wgt * s.red_l[w][g];
+      }
+      if (single) {
+        p.out[qrow * D + e] = num / den;
+      } else {
+        p.ws_o[(size_t)item * G * D + e] = num;
+        if (e % D == 0) p.ws_ml[(size_t)item * G + g] = make_float2(M, den);
+      }
+    }
+    if (!single) {
+      __threadfence();
+      named_bar_sync(1, kWarps * 32);
+      if (tid == 0) s.last = atomicAdd(&p.ctrl[2 + f.group], 1) == f.nch - 1;
+      named_bar_sync(1, kWarps * 32);
+      if (s.last) {
+        __threadfence();
+        if (tid == 0) p.ctrl[2 + f.group] = 0;  // left at zero for the next call
+        for (int e = tid; e < G * D; e += kWarps * 32) {
+          const int g = e / D;
+          float M = -INFINITY;
+          for (int c = 0; c < f.nch; ++c)
+            M = fmaxf(M, __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]).x);
+          float num = 0.f, den = 0.f;
+          for (int c = 0; c < f.nch; ++c) {
+            const float2 ml = __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]);
+            const float wgt = fast_exp2(ml.x - M);
+            den += wgt * ml.y;
+            num += wgt * __ldcg(&p.ws_o[(size_t)(item_base + c) * G * D + e]);
+          }
+          p.out[qrow * D + e] = num / den;
+        }
+      }
+    }
   }
 }
 
@@ -188,6 +554,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int units = p.B * p.Hkv;
 
+  // Launched as a programmatic dependent of the previous step: let the next
+  // step's CTAs take SMs as this grid's CTAs leave, and wait here until the
+  // previous grid has completed and its writes (lengths, appended rows,
+  // counters) are visible.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   // Work list of this step from the current lengths (read once, before any
   // CTA can advance them: that happens after every CTA has exited).
   if (tid < p.L) {
@@ -195,11 +567,11 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     const int len = p.lens[l];
     const bool full = len < 0 || len >= p.cap[l];
     s.len[tid] = full ? -1 : len;
-    s.nch[tid] = full ? 1 : (len + 1 + C::ITEM_ROWS - 1) / C::ITEM_ROWS;
+    s.nch[tid] = full ? 1 : (len + 1 + kItemRows - 1) / kItemRows;
     if (full && blockIdx.x == 0) report(p.status, RIPPLE_EFULL);
   }
   if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < C::STAGES; ++i) {
       mbar_init(&s.full[i], 1);
       mbar_init(&s.empty[i], kWarps);
     }
@@ -207,6 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       mbar_init(&s.item_full[i], 1);
       mbar_init(&s.item_empty[i], kWarps);
     }
+    s.abort_flag = 0;
     fence_mbar_init();
   }
   __syncthreads();
@@ -222,290 +595,13 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   const int total = s.base[p.L];
 
   if (warp == kWarps) {
-    // ------------------------------------------------ producer warp
-    int icount = 0;
-    uint32_t j = 0;
-    int it = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
-    int nxt = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
-    it = __shfl_sync(0xffffffffu, it, 0);
-    nxt = __shfl_sync(0xffffffffu, nxt, 0);
-    for (;;) {
-      const int slot = icount % kItemSlots;
-      mbar_wait(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, p.status);
-      __syncwarp();
-      if (lane == 0) {
-        s.item_id[slot] = it;
-        mbar_arrive(&s.item_full[slot]);
-      }
-      ++icount;
-      if (it >= total) break;
-      // The first sub-chunks of the very first item get an L2 prefetch too.
-      if (lane == 0 && icount == 1)
-        for (int k = 0; k < kPrefetchAhead; ++k) prefetch_sub(p, s, total, it, nxt, k);
-      int nxt2 = lane == 0 ? atomicAdd(&p.ctrl[0], 1) : 0;
-      const ItemInfo f = item_info(p, s, it);
-      if (!f.full) {
-        const int nsub = (f.rows + C::CR - 1) / C::CR;
-        const size_t gbase = (size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer];
-        for (int sub = 0; sub < nsub; ++sub, ++j) {
-          const int stage = j % kStages;
-          mbar_wait(&s.empty[stage], ((j / kStages) & 1) ^ 1, p.status);
-          __syncwarp();
-          const int rs = f.r0 + sub * C::CR;
-          const int re = min(rs + C::CR, f.len);  // rows >= len are not in the cache yet
-          const int nk = re > rs ? re - rs : 0;
-          if (f.len >= rs && f.len < rs + C::CR) {
-            // The new token: into the stage and appended to the cache.
-            const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * C::ROW_BYTES;
-            for (int e = lane; e < 2 * C::NPIECE; e += 32) {
-              const int v = e >= C::NPIECE, pc = e % C::NPIECE;
-              const uint4 val = reinterpret_cast<const uint4 *>(
-                  (const uint8_t *)(v ? p.v_new : p.k_new) + nb)[pc];
-              reinterpret_cast<uint4 *>(s.kv[stage][v] + (size_t)(f.len - rs) * C::ROW_BYTES)[pc] =
-                  val;
-              reinterpret_cast<uint4 *>((uint8_t *)(v ? p.vc[f.layer] : p.kc[f.layer]) +
-                                        (gbase + f.len) * C::ROW_BYTES)[pc] = val;
-            }
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            if (nk > 0) {
-              const size_t off = (gbase + rs) * C::ROW_BYTES;
-              mbar_arrive_expect_tx(&s.full[stage], 2u * nk * C::ROW_BYTES);
-              bulk_g2s(s.kv[stage][0], (const uint8_t *)p.kc[f.layer] + off, nk * C::ROW_BYTES,
-                       &s.full[stage]);
-              bulk_g2s(s.kv[stage][1], (const uint8_t *)p.vc[f.layer] + off, nk * C::ROW_BYTES,
-                       &s.full[stage]);
-            } else {
-              mbar_arrive(&s.full[stage]);
-            }
-            // Keep kPrefetchAhead more sub-chunks on their way into L2.
-            prefetch_sub(p, s, total, it, nxt, sub + kPrefetchAhead);
-          }
-        }
-      }
-      it = nxt;
-      nxt = __shfl_sync(0xffffffffu, nxt2, 0);
-    }
+    if (lane == 0) produce<Tin, D, G>(p, s, total);
   } else {
-    // ------------------------------------------------ compute warps
-    const int slot_l = lane % C::S;            // lane within its row
-    const int hq = slot_l / C::HL;             // head this lane holds after the reduce-scatter
-    const int rw0 = warp * C::RPW;             // this warp's first row in a sub-chunk
-    int icount = 0;
-    uint32_t j = 0;
-    for (;;) {
-      const int slot = icount % kItemSlots;
-      mbar_wait(&s.item_full[slot], (icount / kItemSlots) & 1, p.status);
-      __syncwarp();
-      const int it = s.item_id[slot];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s.item_empty[slot]);
-      ++icount;
-      if (it >= total) break;
-      const ItemInfo f = item_info(p, s, it);
-      const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
-      if (f.full) {
-        for (int e = tid; e < G * D; e += kWarps * 32) p.out[qrow * D + e] = 0.f;
-        continue;
-      }
-      // Query slice (the lane's pieces of each head), pre-scaled to log2 units.
-      float2 q2[G][C::DL / 2];
-      {
-        const Tin *qg = (const Tin *)p.q + qrow * D;
-#pragma unroll
-        for (int g = 0; g < G; ++g)
-#pragma unroll
-          for (int k = 0; k < C::PPL; ++k) {
-            float2 t[C::PE / 2];
-            load_pairs<C::PE / 2>(qg + g * D + (slot_l + k * C::S) * C::PE, t);
-#pragma unroll
-            for (int e = 0; e < C::PE / 2; ++e)
-              q2[g][k * C::PE / 2 + e] = make_float2(t[e].x * p.scale2, t[e].y * p.scale2);
-          }
-      }
-      float2 acc[G][C::DV / 2];
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-#pragma unroll
-        for (int e = 0; e < C::DV / 2; ++e) acc[g][e] = make_float2(0.f, 0.f);
-      float m_run = -INFINITY, l_run = 0.f;  // of head hq, over this warp's rows
-      const int nsub = (f.rows + C::CR - 1) / C::CR;
-
-      for (int sub = 0; sub < nsub; ++sub, ++j) {
-        const int stage = j % kStages;
-        mbar_wait(&s.full[stage], (j / kStages) & 1, p.status);
-        __syncwarp();
-        const int nrows = min(C::CR, f.r0 + f.rows - (f.r0 + sub * C::CR));
-        const Tin *ks = (const Tin *)s.kv[stage][0];
-        const Tin *vs = (const Tin *)s.kv[stage][1];
-
-        // Scores of this warp's rows.
-        float sc[C::NIT];
-#pragma unroll
-        for (int t = 0; t < C::NIT; ++t) {
-          const int row = rw0 + t * C::RPI + lane / C::S;
-          float2 d2[G];
-#pragma unroll
-          for (int g = 0; g < G; ++g) d2[g] = make_float2(0.f, 0.f);
-          if (row < nrows) {
-#pragma unroll
-            for (int k = 0; k < C::PPL; ++k) {
-              float2 kp[C::PE / 2];
-              load_pairs<C::PE / 2>(ks + (size_t)row * D + (slot_l + k * C::S) * C::PE, kp);
-#pragma unroll
-              for (int g = 0; g < G; ++g)
-#pragma unroll
-                for (int e = 0; e < C::PE / 2; ++e)
-                  d2[g] = __ffma2_rn(q2[g][k * C::PE / 2 + e], kp[e], d2[g]);
-            }
-          }
-          float v[G];
-#pragma unroll
-          for (int g = 0; g < G; ++g) v[g] = d2[g].x + d2[g].y;
-          // Reduce-scatter over the S lanes of the row: afterwards every lane
-          // holds the full dot product of head hq.
-          int nv = G;
-#pragma unroll
-          for (int o = C::S / 2; o >= 1; o >>= 1) {
-            if (nv > 1) {
-              const bool upper = (lane & o) != 0;
-              const int half = nv / 2;
-#pragma unroll
-              for (int i = 0; i < G / 2; ++i) {
-                if (i < half) {
-                  const float send = upper ? v[i] : v[i + half];
-                  const float keep = upper ? v[i + half] : v[i];
-                  v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-                }
-              }
-              nv = half;
-            } else {
-              v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-            }
-          }
-          sc[t] = row < nrows ? v[0] : -INFINITY;
-        }
-
-        // Online softmax of head hq over this warp's rows.
-        float mloc = sc[0];
-#pragma unroll
-        for (int t = 1; t < C::NIT; ++t) mloc = fmaxf(mloc, sc[t]);
-#pragma unroll
-        for (int o = C::S; o < 32; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
-        const float mnew = fmaxf(m_run, mloc);
-        const bool any = mnew != -INFINITY;
-        const float alpha = any ? fast_exp2(m_run - mnew) : 1.f;
-        float lsum = 0.f;
-#pragma unroll
-        for (int t = 0; t < C::NIT; ++t) {
-          const float e = any ? fast_exp2(sc[t] - mnew) : 0.f;
-          sc[t] = e;
-          lsum += e;
-        }
-#pragma unroll
-        for (int o = C::S; o < 32; o <<= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
-        l_run = l_run * alpha + lsum;
-        m_run = mnew;
-        if (slot_l % C::HL == 0) {
-#pragma unroll
-          for (int t = 0; t < C::NIT; ++t) s.pw[warp][t * C::RPI + lane / C::S][hq] = sc[t];
-          if (lane < C::S) s.aw[warp][hq] = alpha;
-        }
-        __syncwarp();
-
-        // Output rows of this warp.
-        {
-          float a[G];
-          load_probs<G>(s.aw[warp], a);
-#pragma unroll
-          for (int g = 0; g < G; ++g)
-#pragma unroll
-            for (int e = 0; e < C::DV / 2; ++e) {
-              acc[g][e].x *= a[g];
-              acc[g][e].y *= a[g];
-            }
-          const int rmax = min(C::RPW, nrows - rw0);
-#pragma unroll
-          for (int r = 0; r < C::RPW; ++r) {
-            if (r >= rmax) break;
-            float pr[G];
-            load_probs<G>(s.pw[warp][r], pr);
-            float2 vp[C::DV / 2];
-            load_pairs<C::DV / 2>(vs + (size_t)(rw0 + r) * D + lane * C::DV, vp);
-#pragma unroll
-            for (int g = 0; g < G; ++g)
-#pragma unroll
-              for (int e = 0; e < C::DV / 2; ++e)
-                acc[g][e] = __ffma2_rn(make_float2(pr[g], pr[g]), vp[e], acc[g][e]);
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s.empty[stage]);
-      }
-
-      // Item end: merge the 16 warps' states.
-      if (slot_l % C::HL == 0 && lane < C::S) {
-        s.red_m[warp][hq] = m_run;
-        s.red_l[warp][hq] = l_run;
-      }
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-#pragma unroll
-        for (int e = 0; e < C::DV / 2; ++e)
-          *reinterpret_cast<float2 *>(&s.red_o[warp][g * D + lane * C::DV + 2 * e]) = acc[g][e];
-      named_bar_sync(1, kWarps * 32);
-      const bool single = f.nch == 1;
-      const int item_base = s.base[f.pos] + (f.b * p.Hkv + f.h) * f.nch;
-      const int item = item_base + f.chunk;
-      for (int e = tid; e < G * D; e += kWarps * 32) {
-        const int g = e / D;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, s.red_m[w][g]);
-        float num = 0.f, den = 0.f;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
-          const float wgt = fast_exp2(s.red_m[w][g] - M);
-          num += wgt * s.red_o[w][e];
-          den += wgt * s.red_l[w][g];
-        }
-        if (single) {
-          p.out[qrow * D + e] = num / den;
-        } else {
-          p.ws_o[(size_t)item * G * D + e] = num;
-          if (e % D == 0) p.ws_ml[(size_t)item * G + g] = make_float2(M, den);
-        }
-      }
-      if (!single) {
-        __threadfence();
-        named_bar_sync(1, kWarps * 32);
-        if (tid == 0) s.last = atomicAdd(&p.ctrl[2 + f.group], 1) == f.nch - 1;
-        named_bar_sync(1, kWarps * 32);
-        if (s.last) {
-          __threadfence();
-          for (int e = tid; e < G * D; e += kWarps * 32) {
-            const int g = e / D;
-            float M = -INFINITY;
-            for (int c = 0; c < f.nch; ++c)
-              M = fmaxf(M, __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]).x);
-            float num = 0.f, den = 0.f;
-            for (int c = 0; c < f.nch; ++c) {
-              const float2 ml = __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]);
-              const float wgt = fast_exp2(ml.x - M);
-              den += wgt * ml.y;
-              num += wgt * __ldcg(&p.ws_o[(size_t)(item_base + c) * G * D + e]);
-            }
-            p.out[qrow * D + e] = num / den;
-          }
-        }
-      }
-      named_bar_sync(1, kWarps * 32);  // red_* free for the next item
-    }
+    consume<Tin, D, G>(p, s, total, warp, lane);
   }
 
-  // The last CTA to leave advances the lengths of the layers it could append to.
+  // The last CTA to leave advances the lengths of the layers it appended to
+  // and leaves the item and exit counters at zero for the next call.
   __syncwarp();
   __syncthreads();
   if (tid == 0) {
@@ -513,49 +609,88 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     if (atomicAdd(&p.ctrl[1], 1) == (int)gridDim.x - 1) {
       for (int t = 0; t < p.L; ++t)
         if (s.len[t] >= 0) p.lens[p.order[t]] = s.len[t] + 1;
+      p.ctrl[0] = 0;
+      p.ctrl[1] = 0;
     }
   }
 }
 
-int sm_count_cached() {
-  static int n = 0;
-  if (n == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 1;
+// ------------------------------------------------------------ host side
+
+constexpr int kMaxDevices = 64;
+
+int sm_count(int dev) {
+  static int n[kMaxDevices] = {};
+  if (dev < 0 || dev >= kMaxDevices) return 1;
+  if (n[dev] == 0) {
+    int v = 0;
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    n[dev] = v > 0 ? v : 1;
   }
-  return n;
+  return n[dev];
 }
 
 template <typename Tin, int D, int G>
-cudaError_t launch_g(const DecParams &p, cudaStream_t st) {
+cudaError_t launch_g(const DecParams &p, int dev, cudaStream_t st) {
+  static bool attr_set[kMaxDevices] = {};
   const int smem = (int)sizeof(DecSmem<Tin, D, G>);
-  cudaError_t e = cudaFuncSetAttribute(decode_kernel<Tin, D, G>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-  if (e != cudaSuccess) return e;
-  decode_kernel<Tin, D, G><<<sm_count_cached(), kThreads, smem, st>>>(p);
+  static_assert(sizeof(DecSmem<Tin, D, G>) <= 227 * 1024, "shared memory per CTA");
+  if (!attr_set[dev]) {
+    const cudaError_t e = cudaFuncSetAttribute(decode_kernel<Tin, D, G>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr_set[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sm_count(dev));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, decode_kernel<Tin, D, G>, p);
   count_launches(1);
-  return cudaGetLastError();
+  return e;
 }
 
 template <typename Tin, int D>
-cudaError_t launch_d(const DecParams &p, cudaStream_t st) {
+cudaError_t launch_d(const DecParams &p, int dev, cudaStream_t st) {
   switch (p.G) {
-    case 1: return launch_g<Tin, D, 1>(p, st);
-    case 2: return launch_g<Tin, D, 2>(p, st);
-    case 4: return launch_g<Tin, D, 4>(p, st);
-    case 8: return launch_g<Tin, D, 8>(p, st);
+    case 1: return launch_g<Tin, D, 1>(p, dev, st);
+    case 2: return launch_g<Tin, D, 2>(p, dev, st);
+    case 4: return launch_g<Tin, D, 4>(p, dev, st);
+    case 8: return launch_g<Tin, D, 8>(p, dev, st);
     default: return cudaErrorInvalidValue;
   }
 }
 
-// Cache rows per work item of the kernel that serves this descriptor.
-int item_rows(const ripple_decode_desc *d) {
-  if (decode_tc_supported(d)) return kTcItemRows;
-  const int row_bytes = d->head_dim * (d->dtype == RIPPLE_F32 ? 4 : 2);
-  return (kStageBytes / row_bytes) * kItemSub;
+// Counter blocks left at zero by the previous call on each device: the kernel
+// resets its counters as it exits, so a workspace used by the previous call
+// on the device needs no clearing.
+struct CleanCtrl {
+  const void *ptr = nullptr;
+  size_t bytes = 0;
+};
+CleanCtrl g_clean[kMaxDevices];
+std::mutex g_clean_mu;
+
+cudaError_t clear_ctrl_if_needed(int dev, int *ctrl, size_t bytes, cudaStream_t st) {
+  std::lock_guard<std::mutex> lock(g_clean_mu);
+  CleanCtrl &c = g_clean[dev];
+  if (c.ptr == ctrl && c.bytes >= bytes) return cudaSuccess;
+  const cudaError_t e = cudaMemsetAsync(ctrl, 0, bytes, st);
+  if (e == cudaSuccess) {
+    c.ptr = ctrl;
+    c.bytes = bytes;
+  }
+  return e;
 }
+
+// Cache rows per work item (the workspace holds one partial per item).
+int item_rows(const ripple_decode_desc *) { return kItemRows; }
 
 static size_t round_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -645,16 +780,15 @@ ripple_status prepare(const ripple_decode_desc *desc, const void *q, const void 
 
 ripple_status run(const ripple_decode_desc *desc, const DecParams &p, void *stream) {
   cudaStream_t st = (cudaStream_t)stream;
-  if (decode_tc_supported(desc))
-    return launch_decode_tc(p, ctrl_bytes(desc), st) == cudaSuccess ? RIPPLE_OK : RIPPLE_ECUDA;
-  decode_tc_forget_ctrl(p.ctrl);
-  if (cudaMemsetAsync(p.ctrl, 0, ctrl_bytes(desc), st) != cudaSuccess) return RIPPLE_ECUDA;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RIPPLE_ECUDA;
+  if (clear_ctrl_if_needed(dev, p.ctrl, ctrl_bytes(desc), st) != cudaSuccess) return RIPPLE_ECUDA;
   cudaError_t e;
   if (desc->dtype == RIPPLE_F32)
-    e = desc->head_dim == 64 ? launch_d<float, 64>(p, st) : launch_d<float, 128>(p, st);
+    e = desc->head_dim == 64 ? launch_d<float, 64>(p, dev, st) : launch_d<float, 128>(p, dev, st);
   else
-    e = desc->head_dim == 64 ? launch_d<__nv_bfloat16, 64>(p, st)
-                             : launch_d<__nv_bfloat16, 128>(p, st);
+    e = desc->head_dim == 64 ? launch_d<__nv_bfloat16, 64>(p, dev, st)
+                             : launch_d<__nv_bfloat16, 128>(p, dev, st);
   return e == cudaSuccess ? RIPPLE_OK : RIPPLE_ECUDA;
 }
 
@@ -699,8 +833,7 @@ extern "C" ripple_status ripple_decode_attn(const ripple_decode_desc *desc, cons
 // array below instead of a caller workspace. Every GPU that loads the library
 // keeps it until the process exits; all calls on a device share it. Its
 // counters start at zero (zero-initialised at load) and every call leaves them
-// at zero (the tensor-core kernel resets them as it exits, the other kernels
-// are preceded by a memset on the stream); every partial a call reads it has
+// at zero (the kernel resets them as it exits); every partial a call reads it has
 // rewritten, so no state carries over from the previous call. Calls that
 // overlap on the GPU race on it.
 
@@ -709,7 +842,6 @@ static __device__ __align__(256) float
 
 namespace {
 
-constexpr int kMaxDevices = 256;
 std::mutex g_scratch_mutex;
 float *g_scratch_addr[kMaxDevices] = {};
 

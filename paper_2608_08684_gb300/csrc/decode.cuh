@@ -1,5 +1,5 @@
-// Parameters of one decode step, shared by the decode kernels (SIMT and
-// tensor-core) and their host-side set-up.
+// Parameters of one decode step, shared by the decode kernel and its
+// host-side set-up.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -25,15 +25,6 @@ struct DecParams {
   int order[RIPPLE_MAX_LAYERS];  // layers by decreasing capacity
 };
 
-// Tensor-core decode (bf16, d = 128, up to kTcMaxLayers layers per call).
-constexpr int kTcMaxLayers = 80;
-constexpr int kTcItemRows = 4096;  // cache rows per work item (32 tiles of 128)
-bool decode_tc_supported(const ripple_decode_desc *d);
-// Clears the counter block itself unless the previous tensor-core call on
-// this device left this block at zero.
-cudaError_t launch_decode_tc(const DecParams &p, size_t ctrl_bytes, cudaStream_t st);
-// The counter block at `ctrl` is no longer known to be zero (another kernel
-// used it).
-void decode_tc_forget_ctrl(const void *ctrl);
+constexpr int kItemRows = 4096;  // cache rows per work item
 
 }  // namespace ripple

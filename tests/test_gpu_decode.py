@@ -66,8 +66,7 @@ DECODE_SHAPES = [
                           dtype="bf16", seed=42), [127, 513]),
     ("bf16-d64-G1", dict(n_layers=2, batch=2, n_q_heads=3, n_kv_heads=3, head_dim=64,
                          dtype="bf16", seed=43), [64, 200]),
-    # groups split over several work items (4096 rows on the tensor-core path), item edges
-    # and a ragged tail
+    # groups split over several work items (4096 rows each), item edges and a ragged tail
     ("bf16-d128-G4-split", dict(n_layers=4, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
                                 dtype="bf16", kv_dist="scaled_sinks", seed=47),
      [2047, 4096, 4097, 8300]),
@@ -129,7 +128,7 @@ def test_decode_full_cache_reports_and_skips(lib):
 
 
 def test_decode_full_cache_bf16_d128(lib):
-    # the tensor-core path (bf16, d = 128): a full layer is skipped and reported
+    # bf16, d = 128: a full layer is skipped and reported
     wl = synth.WORKLOADS["tiny"].replace(n_layers=2, dtype="bf16", head_dim=128, n_q_heads=8,
                                          n_kv_heads=2, seed=50)
     caps = [300, 300]

@@ -38,7 +38,7 @@ def _decode_steps(lib, s, stream=None):
 @pytest.mark.parametrize("over", [
     dict(n_layers=3, batch=2, n_q_heads=8, n_kv_heads=2, head_dim=128, dtype="bf16", seed=61),
     dict(n_layers=2, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=64, dtype="f32", seed=62),
-], ids=["tensor-core", "cuda-core"])
+], ids=["bf16-d128", "f32-d64"])
 def test_decode_steps_replay_from_a_graph(lib, over):
     wl = synth.WORKLOADS["tiny"].replace(**over)
     lens0, steps = [5, 300, 129][:wl.n_layers], 4
