@@ -58,6 +58,10 @@ def parse_args():
                     help="time one entry point alone (one layer / one decode step), e.g. "
                          "as a small ncu target; prints one JSON line")
     ap.add_argument("--repeat", type=int, default=10, help="calls timed in --case mode")
+    ap.add_argument("--layers", type=int, default=1,
+                    help="--case compress: compress this many layers in one "
+                         "ripple_compress_layers call (budgets of the largest-budget layers, "
+                         "all reading that layer's K/V so the device footprint stays one layer's)")
     return ap.parse_args()
 
 
@@ -94,15 +98,36 @@ def run_case(args):
         v_out = torch.empty_like(k_out)
         idx = torch.empty(B * Hkv * n, dtype=torch.int32, device=dev)
         nbytes = B * Hkv * d * e * (wl.seq_len + 3 * n) + B * Hq * wl.window * d * e
+        if args.layers > 1:
+            # several layers in one call: the budgets of the args.layers
+            # largest-budget layers, every layer reading the same K/V
+            lay = sorted(range(L), key=lambda i: -budgets[i])[:args.layers]
+            outs = [(torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
+                     torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
+                     torch.empty(B * Hkv * n_keep[i], dtype=torch.int32, device=dev))
+                    for i in lay]
+            tabs = R.CompressTables([q_win] * len(lay), [k] * len(lay), [v] * len(lay),
+                                    [o[0] for o in outs], [o[1] for o in outs],
+                                    [o[2] for o in outs])
+            ws = torch.empty(R.ripple_compress_layers_workspace_bytes(desc, len(lay)),
+                             dtype=torch.uint8, device=dev)
+            nbytes = sum(B * Hkv * d * e * (wl.seq_len + 3 * n_keep[i]) + B * Hq * wl.window * d * e
+                         for i in lay)
         for i in range(args.repeat + 2):
             a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
-            R.ripple_compress_layer(desc, budgets[layer], q_win, k, v, k_out, v_out, idx, ws,
-                                    dev_status=status)
+            if args.layers > 1:
+                R.ripple_compress_layers(desc, [budgets[i] for i in lay], tabs, ws,
+                                         dev_status=status)
+            else:
+                R.ripple_compress_layer(desc, budgets[layer], q_win, k, v, k_out, v_out, idx, ws,
+                                        dev_status=status)
             b_.record()
             if i >= 2:
                 times.append((a, b_))
-        what = f"compress layer {layer} (budget {budgets[layer]}, n {n})"
+        what = (f"compress {len(lay)} layers in one call (budgets of layers {lay}, K/V of "
+                f"layer {layer})" if args.layers > 1 else
+                f"compress layer {layer} (budget {budgets[layer]}, n {n})")
     else:
         steps = args.repeat
         caps = [n + steps + 1 for n in n_keep]

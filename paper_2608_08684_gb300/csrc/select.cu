@@ -1,12 +1,16 @@
 // Pooling of the prefix votes and exact top-k selection per unit (SnapKV's
 // selection rule kept by RippleKV; retained set S_l of Eq. 4).
 //
-// One 1024-thread CTA per unit (b, h):
+// Three kernels, one result (bit for bit): select_unit_kernel (one CTA per
+// unit, launches with many units), select_cluster_kernel (8-CTA clusters per
+// unit, few units) and select_kernel (very long prefixes). The steps, for
+// one unit (b, h):
 //   1. pooled score of every prefix token (max or mean over the clipped
-//      window), mapped to an order-preserving uint32 key, kept in shared
-//      memory when the prefix fits (global scratch otherwise);
-//   2. radix select over the keys, 11 + 11 + 10 bits from the top, finds the
-//      K-th largest key tau and how many keys equal to tau are kept;
+//      window), mapped to an order-preserving uint32 key (in registers, in
+//      shared memory, or in global scratch for very long prefixes);
+//   2. radix select over the keys (4 x 8 bits, or 11 + 11 + 10 bits, from
+//      the top) finds the K-th largest key tau and how many keys equal to
+//      tau are kept;
 //   3. an ordered compaction writes every token with key > tau and the first
 //      tokens with key == tau (lower index wins ties) in ascending order,
 //      followed by the w window positions P..T-1.
@@ -491,12 +495,209 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
   cluster_sync_all();  // no CTA leaves while others may still read its memory
 }
 
+// Prefixes up to kUMaxP tokens: one 1024-thread CTA per unit and no cluster
+// (a launch covers every unit of every layer, so the GPU is filled by units).
+// The pooled keys stay in registers, key j = i * 1024 + thread (i < 32), so
+// that staging, pooling and every radix round read shared memory with
+// consecutive lanes on consecutive words; four radix rounds of 8 bits count
+// into per-warp histograms (no contention between warps); the ordered
+// compaction takes each warp's ballots per row of 1024 keys and one block
+// scan over the (row, warp) counts. Same result as select_kernel, bit for bit.
+constexpr int kUThreads = 1024;
+constexpr int kUWarps = kUThreads / 32;
+constexpr int kUKeys = 32;                    // keys per thread
+constexpr int kUMaxP = kUThreads * kUKeys;
+constexpr int kUBins = 256;
+constexpr int kUMinUnits = 256;               // units per launch for this kernel
+// shared words before the staged votes: per-warp histograms, bin totals,
+// (row, warp) counts, scan scratch and control
+constexpr int kUHead = kUWarps * kUBins + kUBins + kUKeys * kUWarps + 64;
+
+__global__ void __launch_bounds__(kUThreads, 1)
+    select_unit_kernel(LayerGeom g, const float *votes, const __grid_constant__ SelTable tab) {
+  extern __shared__ uint32_t sm[];
+  uint32_t *hist = sm;                                   // [kUWarps][kUBins]
+  int *tot = (int *)(hist + kUWarps * kUBins);           // [kUBins]
+  int *cnt = tot + kUBins;                               // [kUKeys][kUWarps], packed (gt << 16) | eq
+  int *warp_tot = cnt + kUKeys * kUWarps;                // [33]
+  int *ctl = warp_tot + 40;                              // [2]
+  float *vs = reinterpret_cast<float *>(sm + kUHead);    // [P]
+
+  const int unit = blockIdx.x;  // over all layers of the launch
+  const int layer = unit / tab.upl;
+  const int n_keep = tab.n_keep[layer];
+  const int P = g.P, K = n_keep - g.W;
+  const float *v = votes + (size_t)unit * P;
+  int32_t *out = tab.idx[layer] + (size_t)(unit % tab.upl) * n_keep;
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+
+  for (int j = tid; j < g.W; j += kUThreads) out[K + j] = P + j;
+  if (K <= 0) return;
+  if (K >= P) {
+    for (int t = tid; t < P; t += kUThreads) out[t] = t;
+    return;
+  }
+
+  // Votes into shared memory, eight loads of a thread in flight at once.
+#pragma unroll
+  for (int i0 = 0; i0 < kUKeys; i0 += 8) {
+    float x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int j = (i0 + u) * kUThreads + tid;
+      x[u] = j < P ? __ldcg(v + j) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int j = (i0 + u) * kUThreads + tid;
+      if (j < P) vs[j] = x[u];
+    }
+  }
+  __syncthreads();
+
+  // Pooled keys (window clipped to the prefix).
+  const int half = g.pool_kernel / 2;
+  uint32_t key[kUKeys];
+#pragma unroll
+  for (int i = 0; i < kUKeys; ++i) {
+    const int j = i * kUThreads + tid;
+    float r = 0.f;
+    if (j < P) {
+      if (g.pool_type == RIPPLE_POOL_MAX && half == 3 && j >= 3 && j + 3 < P) {
+        // the 7-wide window away from the prefix edges (almost every key)
+        r = fmaxf(fmaxf(fmaxf(vs[j - 3], vs[j - 2]), fmaxf(vs[j - 1], vs[j])),
+                  fmaxf(fmaxf(vs[j + 1], vs[j + 2]), vs[j + 3]));
+      } else if (g.pool_type == RIPPLE_POOL_MAX) {
+        r = vs[j];
+        for (int d = 1; d <= half; ++d) {
+          if (j - d >= 0) r = fmaxf(r, vs[j - d]);
+          if (j + d < P) r = fmaxf(r, vs[j + d]);
+        }
+      } else if (g.pool_type == RIPPLE_POOL_AVG) {
+        float sum = 0.f;
+        int c = 0;
+        for (int d = -half; d <= half; ++d) {
+          const int pos = j + d;
+          if (pos >= 0 && pos < P) {
+            sum = __fadd_rn(sum, vs[pos]);
+            ++c;
+          }
+        }
+        r = __fdiv_rn(sum, (float)c);
+      } else {
+        r = vs[j];
+      }
+    }
+    key[i] = order_key(r);
+  }
+
+  // Radix select of the K-th largest key: 4 rounds of 8 bits from the top.
+  uint32_t prefix = 0, mask = 0;
+  int remaining = K;
+  uint32_t *hw = hist + wid * kUBins;
+  for (int round = 0; round < 4; ++round) {
+    const int shift = 24 - 8 * round;
+#pragma unroll
+    for (int b = lane; b < kUBins; b += 32) hw[b] = 0;
+    __syncwarp();
+#pragma unroll
+    for (int i = 0; i < kUKeys; ++i) {
+      const int j = i * kUThreads + tid;
+      if (j < P && (key[i] & mask) == prefix) atomicAdd(&hw[(key[i] >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid < kUBins) {
+      int sum = 0;
+#pragma unroll 8
+      for (int w = 0; w < kUWarps; ++w) sum += (int)hist[w * kUBins + tid];
+      tot[tid] = sum;
+    }
+    __syncthreads();
+    if (wid == 0) {
+      // lane l holds digits 255 - 8l down to 248 - 8l
+      int c[8], sum = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        c[q] = tot[kUBins - 1 - 8 * lane - q];
+        sum += c[q];
+      }
+      int incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      int above = incl - sum;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (above < remaining && remaining <= above + c[q]) {
+          ctl[0] = kUBins - 1 - 8 * lane - q;
+          ctl[1] = remaining - above;
+        }
+        above += c[q];
+      }
+    }
+    __syncthreads();
+    prefix |= (uint32_t)ctl[0] << shift;
+    mask |= 255u << shift;
+    remaining = ctl[1];
+  }
+  const uint32_t tau = prefix;
+  const int take_eq = remaining;
+
+  // Ordered compaction: per row i of 1024 keys and warp w, the counts of keys
+  // above tau and equal to tau; one block scan over (row, warp) in key order.
+#pragma unroll
+  for (int i = 0; i < kUKeys; ++i) {
+    const int j = i * kUThreads + tid;
+    const int gt = __popc(__ballot_sync(0xffffffffu, j < P && key[i] > tau));
+    const int eq = __popc(__ballot_sync(0xffffffffu, j < P && key[i] == tau));
+    if (lane == 0) cnt[i * kUWarps + wid] = (gt << 16) | eq;
+  }
+  __syncthreads();
+  {
+    int total;
+    const int x = cnt[tid];  // entry (row tid / 32, warp tid % 32)
+    const int off = block_exclusive_scan(x, warp_tot, &total);
+    cnt[tid] = off;
+  }
+  __syncthreads();
+  const uint32_t below = (1u << lane) - 1u;
+#pragma unroll
+  for (int i = 0; i < kUKeys; ++i) {
+    const int j = i * kUThreads + tid;
+    const bool gt = j < P && key[i] > tau, eq = j < P && key[i] == tau;
+    const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
+    const int off = cnt[i * kUWarps + wid];
+    const int g_rank = (off >> 16) + __popc(bg & below);
+    const int e_rank = (off & 0xffff) + __popc(be & below);
+    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = j;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
                           const CompressWs &ws, const int *n_keep, int32_t *const *idx,
                           cudaStream_t st) {
   if (n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorInvalidValue;
+  // One CTA per unit once the launch has enough units to fill the GPU;
+  // fewer units (a single layer) are spread over 8-CTA clusters instead.
+  if (g.P <= kUMaxP && (long long)g.units * n_layers >= kUMinUnits) {
+    SelTable tab;
+    tab.upl = g.units;
+    for (int l = 0; l < n_layers; ++l) {
+      tab.n_keep[l] = n_keep[l];
+      tab.idx[l] = idx[l];
+    }
+    const size_t smem = sizeof(uint32_t) * ((size_t)kUHead + g.P);
+    cudaError_t e = cudaFuncSetAttribute(select_unit_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    select_unit_kernel<<<g.units * n_layers, kUThreads, smem, st>>>(g, votes, tab);
+    count_launches(1);
+    return cudaGetLastError();
+  }
   const int per_cta = ((g.P + kCluster - 1) / kCluster + 31) & ~31;
   if (per_cta <= kCMaxKeys && (long long)g.units * n_layers * kCluster <= 0x7fffffff) {
     SelTable tab;

@@ -110,6 +110,8 @@ def test_tiny_sequences(lib, T, w):
 @pytest.mark.parametrize("units,P,levels,budget", [
     (3, 480, 7, 100), (2, 4000, 50, 1000), (4, 100, 0, 60), (1, 60000, 300, 9000),
     (2, 1025, 1, 500), (1, 5, 2, 10),
+    # >= 256 units: one CTA per unit, keys in registers (prefixes up to 32768)
+    (256, 480, 7, 100), (300, 4001, 50, 1000), (256, 1025, 1, 500), (256, 32768, 1000, 3000),
 ])
 def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget):
     # identical votes on both sides: selection and gather must agree bit for bit
