@@ -5,18 +5,23 @@
 // Same work split as score_tc.cu (one persistent CTA per SM, item i on CTA
 // i mod grid, each CTA running P1(a_k) then P2(a_k-1) in its step k so that
 // keys are re-read from L2 one item after their first read, a publisher warp
-// merging pass-1 row statistics). Both passes compute
-// D[row][key] = Q . K_tile^T with the queries as the A operand in TMEM, so
-// shared memory holds only key tiles (a 6-stage ring) and each MMA reads only
-// its key tile from shared memory. Pass 2's vote of a key is a sum over rows,
-// i.e. over the epilogue threads: each warp reduce-scatters its 32 rows'
-// probabilities with shuffles (every lane ends with 4 keys' sums) and the
-// four warps' sums are added through shared memory.
+// merging pass-1 row statistics). Each pass takes the layout in which its
+// reduction stays inside one thread:
+//   pass 1  D[row][key] = Q . K_tile^T, queries as the A operand in TMEM
+//           (staged there by the epilogue warps); a thread owns a row and
+//           folds its keys into the row's running max and sum;
+//   pass 2  D[key][row] = K_tile . Q^T, key tile as the A operand and the
+//           queries as the B operand in shared memory (one 32 KB buffer,
+//           loaded by TMA per item); a thread owns a key and sums its 128
+//           rows' probabilities, so a key's vote needs no shuffles and no
+//           exchange between warps.
+// TMEM: three 128-column accumulators and two 64-column query slots. Shared
+// memory: a 5-stage key-tile ring and the pass-2 query buffer.
 //
-// Warp roles (352 threads): warp 0 = key-tile producer, warp 1 = MMA issuer
-// and TMEM owner, warps 2-9 = two epilogue warpgroups taking alternate tiles
-// (they also stage each item's queries into TMEM, half of the columns each),
-// warp 10 = publisher of pass-1 results. Every wait is bounded; on timeout the
+// Warp roles (352 threads): warp 0 = key-tile and query producer, warp 1 =
+// MMA issuer and TMEM owner, warps 2-9 = two epilogue warpgroups taking
+// alternate tiles (they also stage each item's queries into TMEM, half of the
+// columns each), warp 10 = publisher of pass-1 results. Every wait is bounded; on timeout the
 // CTA raises RIPPLE_ETIMEOUT, every role leaves its loop and TMEM is released.
 #include <cuda.h>
 #include <math.h>
@@ -34,13 +39,14 @@ constexpr int kTile = 128;                      // keys per tile
 constexpr int kHalfBytes = kTile * 64 * 2;      // one TMA box: 64 dims of 128 keys
 constexpr int kTileBytes = 2 * kHalfBytes;
 constexpr int kThreads = 352;
-constexpr int kNK = 6;                          // key-tile stages
+constexpr int kNK = 5;                          // key-tile stages
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
-constexpr int kNQ = kLag + 2;                   // query slots in TMEM (64 columns each)
-constexpr int kNA = 2;                          // accumulators in TMEM (128 columns each)
+constexpr int kNQ = 2;                          // pass-1 query slots in TMEM (64 columns each)
+constexpr int kNA = 3;                          // accumulators in TMEM (128 columns each)
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 8;
 constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then query slots
+static_assert(kQCol + kNQ * 64 <= 512, "TMEM columns");
 constexpr long long kWaitCycles = 4000000000LL;
 
 struct Tc1Params {
@@ -83,9 +89,7 @@ __device__ __forceinline__ void tiles_of(const Tc1Params &p, const ItemRef &it, 
 // the GPU) stay in L2 and the keys come from DRAM once; a lag of two leaves
 // the other CTAs more time to publish the statistics pass 2 waits for, but
 // its three items per CTA no longer fit in L2 (measured: 3% faster, 1.6x the
-// DRAM reads). kZip takes the two passes' tiles in alternating pairs instead
-// (a steadier mix of DRAM and L2 reads per CTA; measured slower).
-constexpr bool kZip = false;
+// DRAM reads).
 
 struct Step {
   int u1, a0, n1;  // pass 1: unit, first tile, tiles
@@ -116,33 +120,25 @@ __device__ __forceinline__ Step step_of(const Tc1Params &p, int k, int n) {
 // tiles, so that each warpgroup meets every phase of its accumulator slot.
 __device__ __forceinline__ int wg_of(int tc) { return tc & 1; }
 
-// Position j of step s's tile sequence: pass (1 or 2) and tile offset. With
-// kZip, tiles go in pairs P1 P1 P2 P2 P1 P1 ... (each warpgroup then gets
-// both kinds); the longer pass's remaining tiles follow.
+// Position j of step s's tile sequence: its pass-1 tiles, then its pass-2
+// tiles.
 __device__ __forceinline__ void seq_at(const Step &s, int j, int &pass, int &idx) {
-  const int q = kZip ? min(s.n1, s.n2) / 2 : 0;  // pairs of each pass in the zipped part
-  if (j < 4 * q) {
-    const int blk = j >> 1;
-    pass = 1 + (blk & 1);
-    idx = ((blk >> 1) << 1) + (j & 1);
-    return;
-  }
-  j -= 4 * q;
-  const int r1 = s.n1 - 2 * q;
-  pass = j < r1 ? 1 : 2;
-  idx = 2 * q + (j < r1 ? j : j - r1);
+  pass = j < s.n1 ? 1 : 2;
+  idx = j < s.n1 ? j : j - s.n1;
 }
 
 struct Misc {
   uint64_t k_full[kNK], k_empty[kNK], q_full[kNQ], q_empty[kNQ], acc_full[kNA], acc_empty[kNA];
+  uint64_t qs_full, qs_empty;           // pass-2 queries in shared memory
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
   uint32_t tmem_base;
   int abort_flag;
   float2 pstat[kPubSlots][2][128];      // pass-1 row statistics per slot and warpgroup
-  alignas(16) float red[2][2][4][128];  // [warpgroup][tile parity][warp][key] vote partials
+  alignas(16) float offs[2][128];       // per warpgroup: the pass-2 item's row log-normalisers
 };
 
-constexpr int kOffMisc = kNK * kTileBytes;
+constexpr int kOffQs = kNK * kTileBytes;          // pass-2 queries: two 64-dim halves
+constexpr int kOffMisc = kOffQs + kTileBytes;
 constexpr int kSmemBytes = kOffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
@@ -189,23 +185,12 @@ __device__ __forceinline__ void combine(float &m, float &l, float m2, float l2) 
   m = mm;
 }
 
-// One reduce-scatter step over lanes `o` apart: of the 2n values, lanes with
-// bit `o` set keep the upper n, the others the lower n, each adding the
-// partner's copy of the half it keeps.
-template <int N>
-__device__ __forceinline__ void rs_step(float *v, int o, bool up) {
-#pragma unroll
-  for (int i = 0; i < N; ++i) {
-    const float send = up ? v[i] : v[i + N];
-    const float keep = up ? v[i + N] : v[i];
-    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-  }
-}
-
 // Kernel argument: the keys of every layer as 3-D tensor maps [unit][T][128],
-// and the parameters.
+// the window queries of every layer as 2-D maps [B * Hq * W][128], and the
+// parameters.
 struct Tc1Launch {
   CUtensorMap kmap[kCompressMaxLayers];
+  CUtensorMap qmap[kCompressMaxLayers];
   Tc1Params p;
 };
 
@@ -215,6 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ktiles = smem;
+  uint8_t *qsm = smem + kOffQs;
   Misc *ms = (Misc *)(smem + kOffMisc);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = items_of_cta(p);
@@ -232,6 +218,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->acc_full[i], 1);
       mbar_init(&ms->acc_empty[i], 4);
     }
+    mbar_init(&ms->qs_full, 1);
+    mbar_init(&ms->qs_empty, 1);
     for (int i = 0; i < kPubSlots; ++i) {
       mbar_init(&ms->pub_full[i], 8);
       mbar_init(&ms->pub_empty[i], 1);
@@ -253,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------ key-tile producer
     if (lane == 0) {
-      int kcount = 0;
+      int kcount = 0, qcount = 0;
       const uint64_t keep = policy_evict_last(), drop = policy_evict_first();
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
@@ -262,6 +250,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           {
             int pass, s;
             seq_at(st, j, pass, s);
+            if (pass == 2 && s == 0) {
+              // the pass-2 item's queries (rows of its unit) into shared memory
+              if (!wait_bar(&ms->qs_empty, (qcount & 1) ^ 1, ms, p.status)) {
+                ok = false;
+                break;
+              }
+              const int layer = st.u2 / p.upl, local = st.u2 % p.upl;
+              const int b = local / p.Hkv, h = local % p.Hkv;
+              const int qrow0 = (b * p.Hq + h * p.G) * p.W;
+              mbar_arrive_expect_tx(&ms->qs_full, kTileBytes);
+              tma_load_2d(qsm, &lp.qmap[layer], 0, qrow0, &ms->qs_full);
+              tma_load_2d(qsm + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->qs_full);
+              ++qcount;
+            }
             const int unit = pass == 1 ? st.u1 : st.u2;
             const int tt = pass == 1 ? st.a0 + s : st.b0 + s;
             const int ks = kcount % kNK;
@@ -282,23 +284,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       for (int j = max(0, kcount - kNK); j < kcount; ++j)
         mbar_wait(&ms->k_full[j % kNK], (j / kNK) & 1, nullptr, kWaitCycles / 4);
+      if (qcount > 0) mbar_wait(&ms->qs_full, (qcount - 1) & 1, nullptr, kWaitCycles / 4);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int kcount = 0, acount = 0;
+      int kcount = 0, acount = 0, qcount = 0;
       constexpr uint32_t id = idesc_bf16(128, 128);
-      const uint32_t kbase = smem_u32(ktiles);
+      const uint32_t kbase = smem_u32(ktiles), qsbase = smem_u32(qsm);
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
-        const int qs1 = k % kNQ, qs2 = (k + kNQ - kLag) % kNQ;
+        const int qs1 = k % kNQ;
         if (k < n && !wait_bar(&ms->q_full[qs1], (k / kNQ) & 1, ms, p.status)) break;
         for (int j = 0; j < st.len && ok; ++j) {
           {
             int pass, s;
             seq_at(st, j, pass, s);
-            const uint32_t qa = tmem + kQCol + (pass == 1 ? qs1 : qs2) * 64;
+            if (pass == 2 && s == 0) {
+              if (st.n1 > 0) mma_commit(&ms->q_empty[qs1]);  // item k's TMEM queries are free
+              if (!wait_bar(&ms->qs_full, qcount & 1, ms, p.status)) {
+                ok = false;
+                break;
+              }
+            }
+            const uint32_t qa = tmem + kQCol + qs1 * 64;
             const int ks = kcount % kNK, as = acount % kNA;
             if (!wait_bar(&ms->k_full[ks], (kcount / kNK) & 1, ms, p.status) ||
                 !wait_bar(&ms->acc_empty[as], ((acount / kNA) & 1) ^ 1, ms, p.status)) {
@@ -308,17 +318,31 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const uint32_t d = tmem + as * 128;
             const uint32_t ka = kbase + ks * kTileBytes;
+            if (pass == 1) {
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16_tmem_a(d, qa + kk * 8,
-                              sw128_desc(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32), id, kk > 0);
+              for (int kk = 0; kk < 8; ++kk)
+                mma_bf16_tmem_a(d, qa + kk * 8,
+                                sw128_desc(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32), id,
+                                kk > 0);
+            } else {
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk) {
+                const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+                mma_bf16(d, sw128_desc(ka + off), sw128_desc(qsbase + off), id, kk > 0);
+              }
+            }
             mma_commit(&ms->k_empty[ks]);
             mma_commit(&ms->acc_full[as]);
             ++kcount;
             ++acount;
           }
         }
-        if (ok && k >= kLag) mma_commit(&ms->q_empty[qs2]);  // item k - kLag's slot is free
+        if (ok && st.n2 > 0) {
+          mma_commit(&ms->qs_empty);  // the pass-2 queries are free
+          ++qcount;
+        } else if (ok && st.n1 > 0) {
+          mma_commit(&ms->q_empty[qs1]);  // no pass-2 tiles: item k's TMEM queries are free
+        }
       }
       mma_commit(&ms->mma_done);
       mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
@@ -383,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = quarter * 32 + lane;         // window row of this thread
     const int wtid = threadIdx.x - 64 - wg * 128;
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
-    int tcount = 0, wcount = 0;  // tiles seen, tiles this warpgroup took
+    int tcount = 0;  // tiles seen
 
     // Stages item k's window queries into query slot k % kNQ: this thread's
     // row, this warpgroup's half of the 64 columns.
@@ -421,7 +445,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Step st = step_of(p, k, n);
       float m = -INFINITY, l = 0.f;    // pass 1 of item k: this row's max and sum
       const int last_vis = p.P + r % p.W;
-      float off = 0.f;                 // pass 2 of item k - kLag: this row's log-normaliser
       for (int j = 0; j < st.len; ++j) {
         int pass, s;
         seq_at(st, j, pass, s);
@@ -484,51 +507,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (pass == 2) {
           // ---------------- a pass-2 tile of item k - kLag: votes of its keys
+          // (D[key][row]: this thread's TMEM lane is key t * 128 + r)
           if (s == 0) {
             if (wtid == 0) wait_ready(&p.ctrl[p.units + st.u2], ms, p.status);
             named_bar_sync(3 + wg, 128);
-            off = __ldcg(&p.lognorm[(size_t)st.u2 * 128 + r]);
+            ms->offs[wg][wtid] = __ldcg(&p.lognorm[(size_t)st.u2 * 128 + wtid]);
+            named_bar_sync(3 + wg, 128);
           }
           const int t = st.b0 + s;
           const int mine = wg_of(tcount) == wg;
           const int as = tcount % kNA, ph = (tcount / kNA) & 1;
           ++tcount;
-          if (mine) {
-            const bool got = warp_wait(&ms->acc_full[as], ph, ms, p.status);
-            float v[128];
-            if (got) {
-              tc_fence_after();
-              uint32_t x[4][32];
+          if (mine && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
+            tc_fence_after();
+            uint32_t x[4][32];
 #pragma unroll
-              for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + as * 128 + c * 32, x[c]);
-              tmem_wait_ld();
-              tc_fence_before();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + as * 128 + c * 32, x[c]);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+            float sv[8];
 #pragma unroll
-              for (int c = 0; c < 4; ++c)
+            for (int i = 0; i < 8; ++i) sv[i] = 0.f;
+            const float4 *o4 = reinterpret_cast<const float4 *>(ms->offs[wg]);
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  v[c * 32 + j] = fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -off));
-            } else {
+            for (int c = 0; c < 4; ++c)
 #pragma unroll
-              for (int j = 0; j < 128; ++j) v[j] = 0.f;
-            }
-            // Sum over the warp's 32 rows: lane L ends with keys 4L .. 4L + 3.
-            rs_step<64>(v, 16, lane & 16);
-            rs_step<32>(v, 8, lane & 8);
-            rs_step<16>(v, 4, lane & 4);
-            rs_step<8>(v, 2, lane & 2);
-            rs_step<4>(v, 1, lane & 1);
-            float *red = ms->red[wg][wcount & 1][0];
-            *reinterpret_cast<float4 *>(red + quarter * 128 + 4 * lane) =
-                make_float4(v[0], v[1], v[2], v[3]);
-            named_bar_sync(3 + wg, 128);
+              for (int j4 = 0; j4 < 8; ++j4) {
+                const float4 o = o4[c * 8 + j4];
+                const float *x4 = reinterpret_cast<const float *>(&x[c][4 * j4]);
+                sv[(4 * j4) & 7] += fast_exp2(fmaf(x4[0], p.scale2, -o.x));
+                sv[(4 * j4 + 1) & 7] += fast_exp2(fmaf(x4[1], p.scale2, -o.y));
+                sv[(4 * j4 + 2) & 7] += fast_exp2(fmaf(x4[2], p.scale2, -o.z));
+                sv[(4 * j4 + 3) & 7] += fast_exp2(fmaf(x4[3], p.scale2, -o.w));
+              }
             const float vote =
-                (red[wtid] + red[128 + wtid]) + (red[256 + wtid] + red[384 + wtid]);
-            const int key = t * kTile + wtid;
+                ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
+            const int key = t * kTile + r;
             if (key < p.P) p.votes[(size_t)st.u2 * p.P + key] = vote;
-            ++wcount;
           }
         }
       }
@@ -585,6 +602,14 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
     cuuint32_t es[3] = {1, 1, 1};
     if (enc(&lp.kmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k[l]), dims,
             strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    cuuint64_t qdims[2] = {128, (cuuint64_t)g.B * g.Hq * g.W};
+    cuuint64_t qstrides[1] = {256};
+    cuuint32_t qbox[2] = {64, 128};
+    cuuint32_t qes[2] = {1, 1};
+    if (enc(&lp.qmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(q_win[l]), qdims,
+            qstrides, qbox, qes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
