@@ -465,17 +465,19 @@ def run_ours(args, rank, world, local_rank):
                 "kernel": "decode_kernel (ripple_decode_attn, one launch per step)",
                 "bytes_per_launch": round(st.decode_bytes_per_step()),
                 "ms_per_launch": round(dec_avg, 5), "peak_source": hbm_src}
-    comp_traffic = profile_traffic("compress_kernels_llama3-8b_B4_T32768_layer12.md",
+    comp_traffic = profile_traffic("compress_kernels_llama3-8b_B4_T32768_8layers.md",
                                    ["score_tc1.cu", "select.cu", "gather.cu", "tc_ptx.cuh",
                                     "common.cuh"], st.compress_bytes()) \
         if wl.name.startswith("llama3-8b-32L-32q8kv-d128-B4-T32768") else None
     roof_comp = {"bound": "hbm", "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s",
                  "frac": round(comp_gbs / hbm, 4), "traffic": comp_traffic,
-                 "traffic_source": ("ncu dram bytes of the three kernels on the largest-budget "
-                                    "layer (profiles/compress_kernels_llama3-8b_B4_T32768_"
-                                    "layer12.md), scaled to all layers by algorithmic bytes")
+                 "traffic_source": ("ncu dram bytes of the three kernels on an 8-layer "
+                                    "ripple_compress_layers call (profiles/compress_kernels_"
+                                    "llama3-8b_B4_T32768_8layers.md), scaled to all layers by "
+                                    "algorithmic bytes")
                  if comp_traffic else None,
-                 "kernel": "score_tc1_kernel + select_cluster_kernel + gather_kernel (ripple_compress_layer, all layers)",
+                 "kernel": ("score_tc1_kernel + select_unit_kernel + gather_kernel "
+                            "(ripple_compress_layers, all layers in three launches)"),
                  "bytes_per_launch": round(st.compress_bytes()),
                  "ms_per_launch": round(comp_avg, 4), "peak_source": hbm_src}
     dominant = roof_dec if dec_total >= comp_total else roof_comp
