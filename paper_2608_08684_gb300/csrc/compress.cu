@@ -212,25 +212,22 @@ extern "C" ripple_status ripple_compress_layers(
                                   (const int32_t *const *)idx_out_host, n, k_out_host,
                                   v_out_host, cap, dev_status, st));
   } else {
-    // Other shapes: layer by layer (one layer's share of the workspace each).
-    const CompressWs one = carve_compress_ws(g, workspace);
+    // Other shapes: scoring layer by layer (each layer's votes in its part of
+    // the vote array, the scratch of the multi-layer workspace reused), then
+    // one selection and one gather launch for all layers. A layer that keeps
+    // every token needs no votes (the selection writes 0..T-1 for it).
     for (int l = 0; l < n_layers; ++l) {
-      const bool keep_all = n[l] == g.T;
-      if (g.P > 0 && !keep_all) {
-        cudaError_t e =
-            score_tc_supported(g)
-                ? launch_score_tc(g, q_win_host[l], k_host[l], one, one.votes, dev_status, st)
-                : launch_score_simt(g, q_win_host[l], k_host[l], one, one.votes, st);
-        RIPPLE_CUDA_TRY(e);
-      }
-      int32_t *idx = idx_out_host[l];
-      if (keep_all)
-        RIPPLE_CUDA_TRY(launch_iota(g, idx, st));
-      else
-        RIPPLE_CUDA_TRY(launch_select(g, 1, one.votes, one, &n[l], &idx, st));
-      RIPPLE_CUDA_TRY(launch_gather(g, 1, &k_host[l], &v_host[l], &idx_out_host[l], &n[l],
-                                    &k_out_host[l], &v_out_host[l], &cap[l], dev_status, st));
+      if (g.P == 0 || n[l] == g.T) continue;
+      float *votes_l = ws.votes + (size_t)l * g.units * g.P;
+      cudaError_t e = score_tc_supported(g)
+                          ? launch_score_tc(g, q_win_host[l], k_host[l], ws, votes_l, dev_status, st)
+                          : launch_score_simt(g, q_win_host[l], k_host[l], ws, votes_l, st);
+      RIPPLE_CUDA_TRY(e);
     }
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, st));
+    RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
+                                  (const int32_t *const *)idx_out_host, n, k_out_host,
+                                  v_out_host, cap, dev_status, st));
   }
   for (int l = 0; l < n_layers; ++l) n_keep_host[l] = n[l];
   return RIPPLE_OK;

@@ -48,7 +48,7 @@ SHAPES = [
      [0, 31, 32, 200, 968, 10**6]),
     ("bf16-d128-G4-one-tile", dict(n_layers=3, batch=1, n_q_heads=4, n_kv_heads=1,
                                    head_dim=128, seq_len=130, dtype="bf16", seed=22), [40, 98, 129]),
-    # other shapes: layer by layer inside the call
+    # other shapes: scoring layer by layer, one selection and one gather launch for all layers
     ("bf16-d128-G8", dict(n_layers=3, batch=1, n_q_heads=16, n_kv_heads=2, head_dim=128,
                           seq_len=700, dtype="bf16", seed=23), [300, 50, 699]),
     ("f32-d64-G2", dict(n_layers=4, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=64,
