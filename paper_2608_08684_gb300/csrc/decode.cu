@@ -35,6 +35,8 @@
 // last CTA to leave reset them), and each launch is a programmatic dependent
 // of the previous one on the stream: its CTAs take SMs as the previous step's
 // CTAs leave and wait (griddepcontrol.wait) until that step has completed.
+// CTA b's first item is item b, so that before that wait it can already
+// prefetch its first sub-chunks into L2.
 // Every wait is bounded; on timeout the CTA raises RIPPLE_ETIMEOUT and all
 // roles leave their loops together.
 #include <math.h>
@@ -238,10 +240,11 @@ __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &
   using C = DecCfg<Tin, D, G>;
   const int units = p.B * p.Hkv;
   uint32_t j = 0;
-  int it = atomicAdd(&p.ctrl[0], 1);
+  // The first item of CTA b is item b; later ones come from the counter.
+  int it = min((int)blockIdx.x, total);
   for (int icount = 0;; ++icount) {
     const int slot = icount % kItemSlots;
-    const int nxt = it < total ? atomicAdd(&p.ctrl[0], 1) : total;
+    const int nxt = it < total ? atomicAdd(&p.ctrl[0], 1) + (int)gridDim.x : total;
     if (!wait_bar(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, &s.abort_flag, p.status))
       return;
     const int cur = min(it, total);
@@ -546,6 +549,37 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
   }
 }
 
+// Before the previous step has completed: the first sub-chunks of this CTA's
+// first item (item blockIdx.x) into L2, from the lengths as they read now
+// (one less than this step's if the previous step has not yet advanced
+// them; a prefetch is only a hint), so that this step's first loads do not
+// start from DRAM after the previous step's tail.
+template <typename Tin, int D, int G>
+__device__ __forceinline__ void prefetch_first_item(const DecParams &p) {
+  using C = DecCfg<Tin, D, G>;
+  const int units = p.B * p.Hkv;
+  int rest = (int)blockIdx.x;
+  for (int t = 0; t < p.L; ++t) {
+    const int l = p.order[t];
+    const int len = *(volatile const int32_t *)&p.lens[l];
+    const bool full = len < 0 || len >= p.cap[l];
+    const int nch = full ? 1 : (len + 1 + kItemRows - 1) / kItemRows;
+    if (rest >= units * nch) {
+      rest -= units * nch;
+      continue;
+    }
+    if (full) return;
+    const int unit = rest / nch, chunk = rest % nch;
+    const int r0 = chunk * kItemRows, r1 = min(len, r0 + kItemRows);
+    const int rows = min(r1 - r0, C::STAGES * C::CR);
+    if (rows <= 0) return;
+    const size_t off = ((size_t)unit * p.cap[l] + r0) * C::ROW_BYTES;
+    bulk_prefetch_l2((const uint8_t *)p.kc[l] + off, (uint32_t)rows * C::ROW_BYTES);
+    bulk_prefetch_l2((const uint8_t *)p.vc[l] + off, (uint32_t)rows * C::ROW_BYTES);
+    return;
+  }
+}
+
 template <typename Tin, int D, int G>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecParams p) {
   using C = DecCfg<Tin, D, G>;
@@ -559,6 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   // previous grid has completed and its writes (lengths, appended rows,
   // counters) are visible.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (tid == 0) prefetch_first_item<Tin, D, G>(p);
   asm volatile("griddepcontrol.wait;" ::: "memory");
   // Work list of this step from the current lengths (read once, before any
   // CTA can advance them: that happens after every CTA has exited).
