@@ -481,16 +481,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
             if (tmax != -INFINITY) {
               const float mnew = fmaxf(m, tmax * p.scale2);
-              float sv[8];
+              // fp32x2: logits scaled and shifted two at a time, sums in pairs
+              float2 sv[4];
 #pragma unroll
-              for (int i = 0; i < 8; ++i) sv[i] = 0.f;
+              for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
+              const float2 s2 = make_float2(p.scale2, p.scale2), mn2 = make_float2(-mnew, -mnew);
 #pragma unroll
               for (int c = 0; c < 4; ++c)
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                  sv[j & 7] += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
-              const float sum =
-                  ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
+                for (int j = 0; j < 32; j += 2) {
+                  const float2 y = __ffma2_rn(
+                      make_float2(__uint_as_float(x[c][j]), __uint_as_float(x[c][j + 1])), s2, mn2);
+                  sv[(j >> 1) & 3] =
+                      __fadd2_rn(sv[(j >> 1) & 3], make_float2(fast_exp2(y.x), fast_exp2(y.y)));
+                }
+              const float sum = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
+                                ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
               l = l * fast_exp2(m - mnew) + sum;
               m = mnew;
             }
@@ -527,23 +533,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
-            float sv[8];
+            // fp32x2: logits scaled and shifted two at a time, sums in pairs
+            float2 sv[4];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) sv[i] = 0.f;
+            for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
+            const float2 s2 = make_float2(p.scale2, p.scale2);
             const float4 *o4 = reinterpret_cast<const float4 *>(ms->offs[wg]);
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
               for (int j4 = 0; j4 < 8; ++j4) {
                 const float4 o = o4[c * 8 + j4];
-                const float *x4 = reinterpret_cast<const float *>(&x[c][4 * j4]);
-                sv[(4 * j4) & 7] += fast_exp2(fmaf(x4[0], p.scale2, -o.x));
-                sv[(4 * j4 + 1) & 7] += fast_exp2(fmaf(x4[1], p.scale2, -o.y));
-                sv[(4 * j4 + 2) & 7] += fast_exp2(fmaf(x4[2], p.scale2, -o.z));
-                sv[(4 * j4 + 3) & 7] += fast_exp2(fmaf(x4[3], p.scale2, -o.w));
+                const float2 y0 = __ffma2_rn(make_float2(__uint_as_float(x[c][4 * j4]),
+                                                         __uint_as_float(x[c][4 * j4 + 1])),
+                                             s2, make_float2(-o.x, -o.y));
+                const float2 y1 = __ffma2_rn(make_float2(__uint_as_float(x[c][4 * j4 + 2]),
+                                                         __uint_as_float(x[c][4 * j4 + 3])),
+                                             s2, make_float2(-o.z, -o.w));
+                sv[(2 * j4) & 3] =
+                    __fadd2_rn(sv[(2 * j4) & 3], make_float2(fast_exp2(y0.x), fast_exp2(y0.y)));
+                sv[(2 * j4 + 1) & 3] =
+                    __fadd2_rn(sv[(2 * j4 + 1) & 3], make_float2(fast_exp2(y1.x), fast_exp2(y1.y)));
               }
-            const float vote =
-                ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
+            const float vote = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
+                               ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
             const int key = t * kTile + r;
             if (key < p.P) p.votes[(size_t)st.u2 * p.P + key] = vote;
           }
