@@ -107,13 +107,16 @@ def test_tiny_sequences(lib, T, w):
     assert agree >= 0.999 * total
 
 
-@pytest.mark.parametrize("units,P,levels,budget", [
-    (3, 480, 7, 100), (2, 4000, 50, 1000), (4, 100, 0, 60), (1, 60000, 300, 9000),
-    (2, 1025, 1, 500), (1, 5, 2, 10),
+@pytest.mark.parametrize("units,P,levels,budget,pool,kernel", [
+    (3, 480, 7, 100, "max", 7), (2, 4000, 50, 1000, "max", 7), (4, 100, 0, 60, "max", 7),
+    (1, 60000, 300, 9000, "max", 7), (2, 1025, 1, 500, "max", 7), (1, 5, 2, 10, "max", 7),
     # >= 256 units: one CTA per unit, keys in registers (prefixes up to 32768)
-    (256, 480, 7, 100), (300, 4001, 50, 1000), (256, 1025, 1, 500), (256, 32768, 1000, 3000),
+    (256, 480, 7, 100, "max", 7), (300, 4001, 50, 1000, "max", 7), (256, 1025, 1, 500, "max", 7),
+    (256, 32768, 1000, 3000, "max", 7),
+    # the same kernel's other pooling paths: another window, average, none
+    (256, 700, 3, 200, "max", 5), (256, 600, 0, 150, "avg", 7), (256, 480, 20, 100, "none", 7),
 ])
-def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget):
+def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget, pool, kernel):
     # identical votes on both sides: selection and gather must agree bit for bit
     w = 8
     wl = synth.WORKLOADS["tiny"].replace(batch=1, n_q_heads=units, n_kv_heads=units,
@@ -121,7 +124,7 @@ def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget):
     votes = synth.synthetic_votes(31 + P, units, P, levels)
     k = synth.layer_keys(wl, 0)
     v = synth.layer_values(wl, 0)
-    desc = lib.layer_desc(1, units, units, 64, P + w, w, 7, "max", torch.bfloat16)
+    desc = lib.layer_desc(1, units, units, 64, P + w, w, kernel, pool, torch.bfloat16)
     n = lib.ripple_keep_count(budget, P + w, w)
     k_out = torch.zeros(1, units, n, 64, dtype=torch.bfloat16, device=DEV)
     v_out = torch.zeros_like(k_out)
@@ -132,7 +135,7 @@ def test_selection_bit_exact_on_shared_votes(lib, units, P, levels, budget):
     torch.cuda.synchronize()
     idx = idx.view(units, n).cpu().numpy()
     for u in range(units):
-        pooled = O.pool_scores(votes[u].numpy(), 7, "max")
+        pooled = O.pool_scores(votes[u].numpy(), kernel, pool)
         expect = O.select_tokens(pooled, n, P + w, w)
         np.testing.assert_array_equal(idx[u], expect)
         assert torch.equal(k_out[0, u].cpu(), k[0, u][torch.from_numpy(expect)])
