@@ -440,15 +440,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
             if (tmax == -INFINITY) continue;
             const float mnew = fmaxf(m[nr], tmax * p.scale2);
-            float sv[8];
+            // fp32x2: logits scaled and shifted two at a time, sums in pairs
+            float2 sv[4];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) sv[i] = 0.f;
+            for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
+            const float2 s2 = make_float2(p.scale2, p.scale2), mn2 = make_float2(-mnew, -mnew);
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                sv[j & 7] += fast_exp2(fmaf(__uint_as_float(x[c][j]), p.scale2, -mnew));
-            const float s = ((sv[0] + sv[1]) + (sv[2] + sv[3])) + ((sv[4] + sv[5]) + (sv[6] + sv[7]));
+              for (int j = 0; j < 32; j += 2) {
+                const float2 y = __ffma2_rn(
+                    make_float2(__uint_as_float(x[c][j]), __uint_as_float(x[c][j + 1])), s2, mn2);
+                sv[(j >> 1) & 3] =
+                    __fadd2_rn(sv[(j >> 1) & 3], make_float2(fast_exp2(y.x), fast_exp2(y.y)));
+              }
+            const float s = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
+                            ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
             l[nr] = l[nr] * fast_exp2(m[nr] - mnew) + s;
             m[nr] = mnew;
           }
@@ -480,9 +487,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int as = tcount % C::NA;
           if (!warp_wait(&ms->acc_full[as], (tcount / C::NA) & 1, ms, p.status)) continue;
           tc_fence_after();
-          float vs[8];
+          // fp32x2: logits scaled and shifted two at a time, sums in pairs
+          float2 vs[4];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) vs[i] = 0.f;
+          for (int i = 0; i < 4; ++i) vs[i] = make_float2(0.f, 0.f);
+          const float2 s2 = make_float2(p.scale2, p.scale2);
           const uint32_t base = tmem + lane_addr + as * C::ACC_COLS;
 #pragma unroll
           for (int c4 = 0; c4 < NR; ++c4) {
@@ -500,14 +509,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int j = 0; j < 32; j += 4) {
                 const float4 o = off4[(c4 * 128 + c * 32 + j) >> 2];
-                const int h = (j >> 2) & 1;  // two chains per 4 columns: 8 in flight
-                vs[4 * h + 0] += fast_exp2(fmaf(__uint_as_float(x[c][j + 0]), p.scale2, -o.x));
-                vs[4 * h + 1] += fast_exp2(fmaf(__uint_as_float(x[c][j + 1]), p.scale2, -o.y));
-                vs[4 * h + 2] += fast_exp2(fmaf(__uint_as_float(x[c][j + 2]), p.scale2, -o.z));
-                vs[4 * h + 3] += fast_exp2(fmaf(__uint_as_float(x[c][j + 3]), p.scale2, -o.w));
+                const int h = (j >> 1) & 2;  // two pair chains per 4 columns: 4 in flight
+                const float2 y0 = __ffma2_rn(
+                    make_float2(__uint_as_float(x[c][j]), __uint_as_float(x[c][j + 1])), s2,
+                    make_float2(-o.x, -o.y));
+                const float2 y1 = __ffma2_rn(
+                    make_float2(__uint_as_float(x[c][j + 2]), __uint_as_float(x[c][j + 3])), s2,
+                    make_float2(-o.z, -o.w));
+                vs[h] = __fadd2_rn(vs[h], make_float2(fast_exp2(y0.x), fast_exp2(y0.y)));
+                vs[h + 1] = __fadd2_rn(vs[h + 1], make_float2(fast_exp2(y1.x), fast_exp2(y1.y)));
               }
           }
-          const float vote = ((vs[0] + vs[1]) + (vs[2] + vs[3])) + ((vs[4] + vs[5]) + (vs[6] + vs[7]));
+          const float vote = ((vs[0].x + vs[0].y) + (vs[1].x + vs[1].y)) +
+                             ((vs[2].x + vs[2].y) + (vs[3].x + vs[3].y));
           const int key = t * kTile + lrow;
           if (key < p.P) p.votes[(size_t)it.unit * p.P + key] = vote;
         }
