@@ -20,8 +20,9 @@
 //            S lanes of the row group (warp shuffles) that leaves each lane
 //            with the full dot product of one head;
 //   softmax  each (row group, head) keeps its own running max and sum (online
-//            softmax; the max is moved, and the state rescaled, only when a
-//            score exceeds it by more than 2^8, so rescaling is rare);
+//            softmax; scores are in log2 units and the max is moved, and the
+//            state rescaled, only when a score exceeds it by more than 8, a
+//            probability factor of 2^8, so rescaling is rare);
 //            the probability is computed once per head and all-gathered over
 //            the row group (warp shuffles);
 //   output   fp32x2 FMAs of the probabilities with the lane's value dims.
@@ -56,8 +57,9 @@ constexpr int kMaxStageBytes = 32768;         // K (or V) bytes of one sub-chunk
 constexpr int kRowsPerGroup = 4;              // rows per row group and sub-chunk (warp steps)
 constexpr int kItemSlots = 4;
 constexpr int kMaxStages = 6;
-// Lazy rescaling: a running max is only moved when a score exceeds it by more
-// than 2^kRescaleLog2 (probabilities relative to a stale max stay <= 2^8).
+// Lazy rescaling: a running max (log2 units) is only moved when a score
+// exceeds it by more than kRescaleLog2, so probabilities relative to a stale
+// max stay <= 2^kRescaleLog2.
 constexpr float kRescaleLog2 = 8.f;
 constexpr int kSmemBudget = 226 * 1024;
 constexpr int kMiscBytes = 4096;              // barriers, work list, merge statistics
