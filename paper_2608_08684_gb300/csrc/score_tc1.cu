@@ -44,7 +44,7 @@ constexpr int kLag = 1;                         // pass 2 of item k runs in step
 constexpr int kNQ = 2;                          // pass-1 query slots in TMEM (64 columns each)
 constexpr int kNA = 3;                          // accumulators in TMEM (128 columns each)
 constexpr int kPubSlots = 2;
-constexpr int kMinTilesPerItem = 8;
+constexpr int kMinTilesPerItem = 9;
 constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then query slots
 static_assert(kQCol + kNQ * 64 <= 512, "TMEM columns");
 constexpr long long kWaitCycles = 4000000000LL;
