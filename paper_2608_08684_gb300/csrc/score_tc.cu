@@ -46,7 +46,7 @@ constexpr int kHalfBytes = kTile * 64 * 2;      // 64 bf16 columns of 128 rows: 
 constexpr int kTileBytes = 2 * kHalfBytes;      // one 128 x 128 bf16 tile
 constexpr int kThreads = 352;
 constexpr int kPubSlots = 2;
-constexpr int kMinTilesPerItem = 8;
+constexpr int kMinTilesPerItem = 14;
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 // ------------------------------------------------------------ work list
