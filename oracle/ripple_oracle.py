@@ -21,6 +21,9 @@ Paper passages followed:
     selection rule and only changes b_l. SnapKV (Sec. 2) scores prompt tokens
     from an observation window at the end of the prompt.
   * Sec. 4.1: during decoding each new query attends to the cached states.
+  * Sec. 4.3 (sensitivity profiling, offline): the norm-adaptive Value
+    perturbation (Eq. 6), the output KL averaged over the evaluation window
+    (Eq. 7) and the average over the calibration set (Eq. 8).
 
 Readings where the paper is silent (each is also listed in the design notes):
   R1 Eq. 9 without the +epsilon of Algorithm 1: the only role of epsilon is
@@ -48,6 +51,13 @@ Readings where the paper is silent (each is also listed in the design notes):
   R9 decoding: the new key/value row is appended first and the new query
      attends to it as well (causal self-inclusion); no positional rotation
      (the synthetic keys stand for post-rotation keys).
+  R10 perturbation (Eq. 6): the positions the base method protects (SnapKV's
+     observation window) are left out by the caller through a position
+     range [pos_begin, pos_end) of eligible rows; the draws eps ~ N(0, I) are
+     an input (one d-vector per eligible row), not drawn here.
+  R11 window KL (Eq. 7): P_t and Q_t are the softmax over the vocabulary of
+     the reference and perturbed logits at window position t; logits are
+     finite.
 
 Parity pins (tests/test_oracle_*.py): allocation invariants the paper states
 (sum = B, uniform profile, r = 1, max/min = r, monotonicity, affine
@@ -56,7 +66,9 @@ example; scoring closed forms (identical keys, probability mass per row),
 causal-mask isolation and a loop-level brute force on tiny inputs; pooling
 against scipy's maximum_filter1d; selection against the defining top-k
 property; decoding against torch's scaled_dot_product_attention and the
-len-1 / identical-key closed forms. The end-to-end quality of the method on
+len-1 / identical-key closed forms; perturbation against the one-hot closed
+form and the noise-norm identity; window KL against the two-category and
+uniform-versus-spike closed forms, KL(P||P) = 0 and shift invariance. The end-to-end quality of the method on
 LongBench is parity unpinned (no model weights or dataset here).
 """
 from __future__ import annotations
@@ -245,3 +257,57 @@ def decode_attention(q, k_rows, v_rows, scale):
     m = logits.max(axis=1, keepdims=True)
     e = np.exp(logits - m)
     return (e @ v_rows) / e.sum(axis=1, keepdims=True)
+
+
+# ---------------------------------------------------------------------------
+# Sensitivity profiling, offline (Sec. 4.3, Eqs. 6-8; readings R10, R11).
+# The model forwards between the perturbation and the KL (the "PerturbedPredict"
+# and "ReferencePredict" steps of Algorithm 1) are not part of this oracle.
+# ---------------------------------------------------------------------------
+
+
+def perturb_values(v, eps, alpha, pos_begin, pos_end):
+    """Eq. 6: v~_u = v_u + alpha * ||v_u||_2 * eps_u for every (batch, kv head)
+    and every eligible position u in [pos_begin, pos_end); all other rows are
+    returned unchanged (reading R10).
+
+    v: [B][Hkv][T][d] the layer's Value cache; eps: [B][Hkv][pos_end - pos_begin][d]
+    the standard normal draws, eps[b, h, u - pos_begin] for position u.
+    Returns a float64 copy of v with the eligible rows perturbed.
+    """
+    out = np.array(v, dtype=np.float64, copy=True)
+    rows = out[:, :, pos_begin:pos_end, :]
+    norm = np.sqrt(np.sum(rows * rows, axis=-1, keepdims=True))  # ||v_u||_2 per row
+    out[:, :, pos_begin:pos_end, :] = rows + alpha * norm * np.asarray(eps, dtype=np.float64)
+    return out
+
+
+def log_softmax(x):
+    """log of the softmax over the last axis: x - (m + log sum exp(x - m))."""
+    x = np.asarray(x, dtype=np.float64)
+    m = x.max(axis=-1, keepdims=True)
+    return x - (m + np.log(np.sum(np.exp(x - m), axis=-1, keepdims=True)))
+
+
+def window_kl(p_logits, q_logits):
+    """Eq. 7: d = (1/|W|) sum over window positions t of KL(P_t || Q_t), with
+    P_t = softmax(p_logits[t]) the reference distribution and Q_t =
+    softmax(q_logits[t]) the distribution after the perturbation (reading R11).
+
+    p_logits, q_logits: [|W|][V]. Returns (kl [|W|], d), float64.
+    """
+    log_p = log_softmax(p_logits)
+    log_q = log_softmax(q_logits)
+    kl = np.sum(np.exp(log_p) * (log_p - log_q), axis=-1)
+    return kl, float(np.mean(kl))
+
+
+def sensitivity_profile(d):
+    """Eq. 8: s_l = (1/N) sum_i d_{i,l}; d: [N][|A|] window responses of the N
+    calibration examples for every compressible layer. Returns [|A|] float64,
+    summed in example order."""
+    d = np.asarray(d, dtype=np.float64)
+    s = np.zeros(d.shape[1])
+    for i in range(d.shape[0]):
+        s = s + d[i]
+    return s / d.shape[0]
