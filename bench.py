@@ -54,9 +54,13 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU seconds of the oracle sample")
-    ap.add_argument("--case", choices=["compress", "decode"], default=None,
-                    help="time one entry point alone (one layer / one decode step), e.g. "
-                         "as a small ncu target; prints one JSON line")
+    ap.add_argument("--case", choices=["compress", "decode", "perturb", "kl"], default=None,
+                    help="time one entry point alone (one layer / one decode step / the "
+                         "profiling kernels: Eq. 6 perturbation of one layer's V cache, Eq. 7 "
+                         "window KL of every layer's perturbed run), e.g. as a small ncu "
+                         "target; prints one JSON line")
+    ap.add_argument("--vocab", type=int, default=128256,
+                    help="--case kl: vocabulary size (128256: Llama-3)")
     ap.add_argument("--repeat", type=int, default=10, help="calls timed in --case mode")
     ap.add_argument("--layers", type=int, default=1,
                     help="--case compress: compress this many layers in one "
@@ -85,6 +89,8 @@ def run_case(args):
     n_keep = [R.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets]
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     times = []
+    if args.case in ("perturb", "kl"):
+        return run_profile_case(args, R, synth, wl, dev)
     if args.case == "compress":
         layer = max(range(L), key=lambda i: budgets[i])
         q_win = synth.layer_window_queries(wl, layer, dev)
@@ -165,6 +171,53 @@ def run_case(args):
     hbm, src = measured_peaks()
     gbs = nbytes / (ms / 1e3) / 1e9
     print(json.dumps({"case": args.case, "workload": wl.name, "what": what, "calls": args.repeat if args.case == "decode" else len(times),
+                      "ms_per_call": round(ms, 5), "bytes_per_call": nbytes,
+                      "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
+                      "peak_source": src}), flush=True)
+
+
+def run_profile_case(args, R, synth, wl, dev):
+    """The offline profiling kernels on the workload's shapes (Sec. 4.3):
+    perturb = Eq. 6 on one layer's whole V cache (B, Hkv, T, d of the
+    workload; the observation window protected), out of place;
+    kl = Eq. 7 for n_layers perturbed runs (one per layer) against the
+    reference, over a window of `window` positions and --vocab fp32 logits.
+    Inputs exceed L2 (129 MB), so calls need no flush in between."""
+    import torch
+    B, Hkv, T, d, e = wl.batch, wl.n_kv_heads, wl.seq_len, wl.head_dim, wl.elem_bytes
+    if args.case == "perturb":
+        pb, pe, alpha = 0, T - wl.window, 0.05
+        v = synth.layer_values(wl, 0, dev)
+        eps = synth.perturb_draws(wl, 0, pe - pb, dev)
+        out = torch.empty_like(v)
+        call = lambda: R.ripple_perturb_values(v, eps, alpha, pb, pe, v_out=out)
+        nbytes = 2 * B * Hkv * T * d * e + B * Hkv * (pe - pb) * d * 4
+        what = (f"Eq. 6 on one layer's V cache [{B}][{Hkv}][{T}][{d}] {wl.dtype}, positions "
+                f"[{pb}, {pe}) perturbed, out of place")
+    else:
+        n_sets, n_pos, vocab = wl.n_layers, wl.window, args.vocab
+        p, q = synth.window_logits(wl.seed, n_sets, n_pos, vocab, torch.float32, dev)
+        ws = torch.empty(R.ripple_window_kl_workspace_bytes(n_sets, n_pos, vocab),
+                         dtype=torch.uint8, device=dev)
+        d_out = torch.empty(n_sets, device=dev)
+        kl_out = torch.empty(n_sets, n_pos, device=dev)
+        call = lambda: R.ripple_window_kl(p, q, ws, d_out, kl_out)
+        nbytes = (n_sets + 1) * n_pos * vocab * 4 + (n_sets * n_pos + n_sets) * 4
+        what = (f"Eq. 7 for {n_sets} perturbed runs x {n_pos} window positions x {vocab} "
+                f"fp32 logits")
+    times = []
+    for i in range(args.repeat + 2):
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        call()
+        b_.record()
+        if i >= 2:
+            times.append((a, b_))
+    torch.cuda.synchronize()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in times)
+    hbm, src = measured_peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    print(json.dumps({"case": args.case, "workload": wl.name, "what": what, "calls": len(times),
                       "ms_per_call": round(ms, 5), "bytes_per_call": nbytes,
                       "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
                       "peak_source": src}), flush=True)

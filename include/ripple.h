@@ -8,7 +8,10 @@
  * implements that path: a host budget allocator (Sec. 4.4, Eqs. 9-12), a
  * per-layer compression chain on the GPU (scoring, pooling, top-k selection,
  * gather into a compact cache; Sec. 4.1 Eq. 4 and Sec. 4.4 last paragraph) and
- * GQA decode attention over the ragged compressed caches (Sec. 4.1).
+ * GQA decode attention over the ragged compressed caches (Sec. 4.1); and, for
+ * the offline profile the allocator takes, the Value perturbation and the
+ * window KL divergence on the GPU and the calibration average (Sec. 4.3,
+ * Eqs. 6-8).
  *
  * Conventions for every entry point:
  *   - Pointers named *_host are host memory; every other data pointer is CUDA
@@ -319,6 +322,101 @@ ripple_status ripple_decode_attn_noalloc(const ripple_decode_desc *desc, const v
                                          void *const *k_caches_host, void *const *v_caches_host,
                                          const int32_t *caps_host, int32_t *lens, float *out,
                                          int32_t *dev_status, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Sensitivity profiling (offline; Sec. 4.3, Algorithm 1 "Sensitivity        */
+/* Profiling"). The model forwards that turn a perturbed cache into output    */
+/* logits belong to the caller; these calls cover the perturbation (Eq. 6),   */
+/* the window divergence (Eq. 7) and the calibration average (Eq. 8).         */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+  int32_t batch;      /* B >= 1 */
+  int32_t n_kv_heads; /* Hkv >= 1 */
+  int32_t seq_len;    /* T >= 1, cached positions per (batch, kv head) */
+  int32_t head_dim;   /* d: 64 or 128 */
+  int32_t dtype;      /* ripple_dtype of v and v_out */
+} ripple_cache_desc;
+
+/*
+ * ripple_perturb_values -- norm-adaptive perturbation of one layer's Value
+ * cache (Sec. 4.3, Eq. 6).
+ *
+ * For every batch row b, KV head h and eligible position u in
+ * [pos_begin, pos_end):
+ *   v~_u = v_u + alpha * ||v_u||_2 * eps_u,   eps_u ~ N(0, I) (given),
+ * the norm taken over the d channels of the stored row. The positions the
+ * base compression method protects are excluded by the range (SnapKV protects
+ * its observation window, the last w cached positions: pos_end = T - w). Keys
+ * and other layers are not touched by the method, and not by this call.
+ *
+ * v          [B][Hkv][T][d] the layer's Value cache
+ * eps        fp32 [B][Hkv][pos_end - pos_begin][d] standard normal draws; row
+ *            u - pos_begin belongs to position u. May be NULL when the range
+ *            is empty.
+ * alpha      perturbation strength, finite, >= 0
+ * pos_begin, pos_end  0 <= pos_begin <= pos_end <= T
+ * v_out      [B][Hkv][T][d]: the eligible rows receive v~ rounded to nearest
+ *            (even) in dtype, the other rows a copy of v. v_out == v perturbs
+ *            in place and writes only the eligible rows; any other overlap of
+ *            v_out with v or eps is invalid.
+ * Arithmetic is fp32. The call may be captured in a CUDA graph.
+ * Errors: RIPPLE_EINVAL (bad desc or range, alpha < 0 or not finite, NULL or
+ * not 16-byte aligned pointers), RIPPLE_ECUDA.
+ */
+ripple_status ripple_perturb_values(const ripple_cache_desc *desc, const void *v,
+                                    const float *eps, float alpha, int32_t pos_begin,
+                                    int32_t pos_end, void *v_out, void *stream);
+
+/* Device workspace bytes ripple_window_kl needs for this shape. */
+ripple_status ripple_window_kl_workspace_bytes(int32_t n_sets, int32_t n_pos, int32_t vocab,
+                                               size_t *bytes_host);
+
+/*
+ * ripple_window_kl -- output divergence averaged over the evaluation window
+ * (Sec. 4.3, Eq. 7), for n_sets perturbed runs against one reference run
+ * (set s is typically the run with layer s perturbed).
+ *
+ * For every set s and window position t < n_pos, with P_t = softmax over the
+ * vocabulary of p_logits[t] and Q_{s,t} = softmax of q_logits[s][t]:
+ *   KL_{s,t} = sum_v P_t(v) (log P_t(v) - log Q_{s,t}(v))
+ *   d_s      = (1 / n_pos) sum_t KL_{s,t}
+ *
+ * p_logits   [n_pos][vocab] reference logits (intact cache), finite
+ * q_logits   [n_sets][n_pos][vocab] logits after the perturbation, finite
+ * vocab      >= 1, a multiple of 8 (rows start on 16-byte boundaries)
+ * dtype      ripple_dtype of both logit arrays
+ * kl_out     fp32 [n_sets][n_pos] per-position divergences, or NULL
+ * d_out      fp32 [n_sets] window averages
+ * workspace  device scratch of at least ripple_window_kl_workspace_bytes
+ *            bytes, 256-byte aligned, no initialisation needed
+ * Each row is cut into fixed slices of 8192 logits; a slice is reduced in
+ * fp32 to (max, sum of exponentials, P-weighted logit difference) for p and
+ * (max, sum) for q, the slices of a row are merged in a fixed order and the
+ * divergence is formed in double, so results do not depend on the GPU or on
+ * the run. Identical p and q rows give exactly 0. The call may be captured
+ * in a CUDA graph.
+ * Errors: RIPPLE_EINVAL (n_sets < 1, n_pos < 1, bad vocab or dtype, NULL or
+ * misaligned pointers), RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status:
+ * RIPPLE_ETIMEOUT (a bounded in-kernel wait ran out).
+ */
+ripple_status ripple_window_kl(const void *p_logits, const void *q_logits, int32_t n_sets,
+                               int32_t n_pos, int32_t vocab, int32_t dtype, float *kl_out,
+                               float *d_out, void *workspace, size_t workspace_bytes,
+                               int32_t *dev_status, void *stream);
+
+/*
+ * ripple_sensitivity_profile -- calibration average (Sec. 4.3, Eq. 8), host:
+ *   s_l = (1 / N) sum_i d_{i,l},
+ * summed in example order in double. The result feeds ripple_alloc_budgets.
+ *
+ * d_host     [n_examples][n_layers] window divergences d_{i,l} (Eq. 7), finite
+ * s_host     [n_layers] output
+ * Returns RIPPLE_EINVAL for NULL pointers, n_examples < 1, n_layers < 1 or a
+ * non-finite d. Pure, reentrant, no CUDA calls.
+ */
+ripple_status ripple_sensitivity_profile(const double *d_host, int32_t n_examples,
+                                         int32_t n_layers, double *s_host);
 
 /* Number of kernels this library has launched in this process so far
  * (host-side count of launch calls; for benchmarks and launch accounting). */

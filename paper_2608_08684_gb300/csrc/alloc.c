@@ -1,6 +1,7 @@
 /*
  * Host budget allocator: Sec. 4.4 and Algorithm 1 "Budget Allocation" of the
- * RippleKV paper (Eqs. 9-12, constrained by Eq. 5).
+ * RippleKV paper (Eqs. 9-12, constrained by Eq. 5), and the calibration
+ * average that produces its input profile (Sec. 4.3, Eq. 8).
  *
  * Compiled with -ffp-contract=off: every product and sum is rounded on its
  * own, so the result does not depend on whether the host has fused
@@ -83,6 +84,21 @@ ripple_status ripple_alloc_budgets(const double *sens_host, int32_t n_layers, do
     if (rank < left) budgets_host[l] += 1;
   }
   free(w);
+  return RIPPLE_OK;
+}
+
+/* Eq. 8: s_l = (1/N) sum_i d_{i,l}, accumulated in example order. */
+ripple_status ripple_sensitivity_profile(const double *d_host, int32_t n_examples,
+                                         int32_t n_layers, double *s_host) {
+  if (d_host == NULL || s_host == NULL || n_examples < 1 || n_layers < 1) return RIPPLE_EINVAL;
+  const size_t total = (size_t)n_examples * (size_t)n_layers;
+  for (size_t j = 0; j < total; ++j)
+    if (!isfinite(d_host[j])) return RIPPLE_EINVAL;
+  for (int32_t l = 0; l < n_layers; ++l) {
+    double acc = 0.0;
+    for (int32_t i = 0; i < n_examples; ++i) acc += d_host[(size_t)i * n_layers + l];
+    s_host[l] = acc / (double)n_examples;
+  }
   return RIPPLE_OK;
 }
 

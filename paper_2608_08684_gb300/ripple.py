@@ -49,6 +49,12 @@ class DecodeDesc(ctypes.Structure):
                 ("scale", ctypes.c_float)]
 
 
+class CacheDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("seq_len", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("dtype", ctypes.c_int32)]
+
+
 _p = ctypes.c_void_p
 _i32, _i64, _f64, _sz = ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_size_t
 
@@ -85,6 +91,16 @@ _lib.ripple_decode_attn_noalloc.argtypes = [ctypes.POINTER(DecodeDesc), _p, _p, 
                                             ctypes.POINTER(_p), ctypes.POINTER(_p),
                                             ctypes.POINTER(_i32), _p, _p, _p, _p]
 _lib.ripple_decode_attn_noalloc.restype = _i32
+_lib.ripple_perturb_values.argtypes = [ctypes.POINTER(CacheDesc), _p, _p, ctypes.c_float, _i32,
+                                       _i32, _p, _p]
+_lib.ripple_perturb_values.restype = _i32
+_lib.ripple_window_kl_workspace_bytes.argtypes = [_i32, _i32, _i32, ctypes.POINTER(_sz)]
+_lib.ripple_window_kl_workspace_bytes.restype = _i32
+_lib.ripple_window_kl.argtypes = [_p, _p, _i32, _i32, _i32, _i32, _p, _p, _p, _sz, _p, _p]
+_lib.ripple_window_kl.restype = _i32
+_lib.ripple_sensitivity_profile.argtypes = [ctypes.POINTER(_f64), _i32, _i32,
+                                            ctypes.POINTER(_f64)]
+_lib.ripple_sensitivity_profile.restype = _i32
 _lib.ripple_kernel_launches.argtypes = []
 _lib.ripple_kernel_launches.restype = ctypes.c_uint64
 _lib.ripple_status_string.argtypes = [_i32]
@@ -265,6 +281,55 @@ def ripple_decode_attn_noalloc(desc: DecodeDesc, q, k_new, v_new, tables: Decode
                                            tables.k, tables.v, tables.caps, _ptr(lens),
                                            _ptr(out), _ptr(dev_status), _stream(stream)),
            "ripple_decode_attn_noalloc")
+
+
+# ----------------------------------------------------- sensitivity profiling
+
+
+def ripple_perturb_values(v, eps, alpha: float, pos_begin: int, pos_end: int, v_out=None,
+                          stream=None):
+    """Eq. 6 on one layer's Value cache v [B][Hkv][T][d]: rows in
+    [pos_begin, pos_end) get v + alpha * ||v||_2 * eps (eps fp32
+    [B][Hkv][pos_end - pos_begin][d]). In place when v_out is None, else into
+    v_out (the other rows copied)."""
+    B, H, T, d = v.shape
+    desc = CacheDesc(B, H, T, d, _DTYPES[v.dtype])
+    out = v if v_out is None else v_out
+    _check(_lib.ripple_perturb_values(ctypes.byref(desc), _ptr(v), _ptr(eps), float(alpha),
+                                      int(pos_begin), int(pos_end), _ptr(out), _stream(stream)),
+           "ripple_perturb_values")
+
+
+def ripple_window_kl_workspace_bytes(n_sets: int, n_pos: int, vocab: int) -> int:
+    out = _sz()
+    _check(_lib.ripple_window_kl_workspace_bytes(int(n_sets), int(n_pos), int(vocab),
+                                                 ctypes.byref(out)),
+           "ripple_window_kl_workspace_bytes")
+    return out.value
+
+
+def ripple_window_kl(p_logits, q_logits, workspace, d_out, kl_out=None, dev_status=None,
+                     stream=None):
+    """Eq. 7 for every set s: d_out[s] = mean over window positions t of
+    KL(softmax(p_logits[t]) || softmax(q_logits[s][t])); p_logits [n_pos][V],
+    q_logits [n_sets][n_pos][V] (same dtype), kl_out [n_sets][n_pos] or None."""
+    n_sets, n_pos, vocab = q_logits.shape
+    if tuple(p_logits.shape) != (n_pos, vocab) or p_logits.dtype != q_logits.dtype:
+        raise ValueError("p_logits must be [n_pos][vocab] with q_logits' dtype")
+    _check(_lib.ripple_window_kl(_ptr(p_logits), _ptr(q_logits), n_sets, n_pos, vocab,
+                                 _DTYPES[q_logits.dtype], _ptr(kl_out), _ptr(d_out),
+                                 _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                 _ptr(dev_status), _stream(stream)),
+           "ripple_window_kl")
+
+
+def ripple_sensitivity_profile(d) -> list:
+    """Eq. 8 (host C): s_l = mean over the calibration examples of d[i][l]."""
+    n, L = len(d), len(d[0]) if len(d) else 0
+    flat = (_f64 * (n * L))(*[float(x) for row in d for x in row])
+    out = (_f64 * max(L, 1))()
+    _check(_lib.ripple_sensitivity_profile(flat, n, L, out), "ripple_sensitivity_profile")
+    return [float(out[i]) for i in range(L)]
 
 
 def ripple_kernel_launches() -> int:

@@ -16,6 +16,11 @@ backbones on LongBench, none of which exist here):
   +3 c (attention-sink keys); V, window queries and decode queries ~ N(0, 1);
   decode keys N(0, 1) * c (same channel scales, no sink shift);
 * values are drawn in fp32 and rounded to nearest-even into the workload dtype;
+* profiling inputs (the stand-in for one calibration example's outputs):
+  perturbation draws eps ~ N(0, 1) in fp32; reference logits over a
+  vocabulary = 2.5 N(0, 1) with +12 added to four random tokens per position
+  (a peaked next-token distribution), and the logits of perturbed run s =
+  reference + sigma_s N(0, 1), sigma_s from 0.02 to 0.3 across the sets;
 * layer sensitivity profiles follow the shape the paper reports for
   Llama-3.1-8B (Sec. 3.1: maximum at an intermediate layer, ~18x spread):
   "bump" = a mid-depth Gaussian bump times lognormal(0, 0.3) noise,
@@ -40,7 +45,7 @@ def _splitmix64(x: int) -> int:
 
 
 _TAGS = {"k": 1, "v": 2, "q_win": 3, "scale": 4, "dq": 5, "dk": 6, "dv": 7, "sens": 8,
-         "votes": 9, "ck": 10, "cv": 11}
+         "votes": 9, "ck": 10, "cv": 11, "eps": 12, "lp": 13, "lq": 14}
 
 
 def stream_seed(seed: int, tag: str, layer: int = 0, step: int = 0) -> int:
@@ -236,3 +241,31 @@ def decode_caches(wl: Workload, layer: int, cap: int, device="cpu"):
         k.mul_(channel_scales(wl, layer, device)[None, :, None, :])
     v = _normal(shape, _generator(device, wl.seed, "cv", layer), device)
     return k.to(wl.torch_dtype), v.to(wl.torch_dtype)
+
+
+def perturb_draws(wl: Workload, layer: int, n_rows: int, device="cpu") -> torch.Tensor:
+    """fp32 [B][Hkv][n_rows][d] standard normal draws for one layer's Value
+    perturbation (one d-vector per eligible position)."""
+    shape = (wl.batch, wl.n_kv_heads, n_rows, wl.head_dim)
+    return _normal(shape, _generator(device, wl.seed, "eps", layer), device)
+
+
+def window_logits(seed: int, n_sets: int, n_pos: int, vocab: int, dtype=torch.float32,
+                  device="cpu", sigmas=None):
+    """(p [n_pos][vocab], q [n_sets][n_pos][vocab]) synthetic output logits of a
+    reference run and of n_sets perturbed runs over an evaluation window.
+
+    p = 2.5 N(0, 1) with +12 on four random tokens per position; q[s] = p +
+    sigma_s N(0, 1), sigma_s spaced from 0.02 to 0.3 unless given.
+    """
+    g = _generator(device, seed, "lp")
+    p = 2.5 * _normal((n_pos, vocab), g, device)
+    top = torch.randint(0, vocab, (n_pos, 4), generator=g, device=device)
+    p.scatter_add_(1, top, torch.full((n_pos, 4), 12.0, device=device))
+    if sigmas is None:
+        sigmas = [0.02 + 0.28 * s / max(1, n_sets - 1) for s in range(n_sets)]
+    gq = _generator(device, seed, "lq")
+    q = torch.empty((n_sets, n_pos, vocab), device=device, dtype=torch.float32)
+    for s in range(n_sets):
+        q[s] = p + float(sigmas[s]) * _normal((n_pos, vocab), gq, device)
+    return p.to(dtype), q.to(dtype)

@@ -129,3 +129,45 @@ def test_compress_layers_host_validation(lib):
     st = raw.ripple_compress_layers(ctypes.byref(d), 2, None, None, None, None, None, None,
                                     None, None, n, None, 0, None, None)
     assert st == lib.EINVAL
+
+
+def test_sensitivity_profile_bit_exact_vs_oracle(lib):
+    rnd = random.Random(11)
+    for _ in range(50):
+        n, L = rnd.randint(1, 9), rnd.choice([1, 4, 32, 80])
+        d = [[rnd.lognormvariate(-5.0, 1.5) for _ in range(L)] for _ in range(n)]
+        assert lib.ripple_sensitivity_profile(d) == [float(x) for x in O.sensitivity_profile(d)]
+    raw = lib._lib
+    out = (ctypes.c_double * 2)()
+    bad = (ctypes.c_double * 2)(1.0, math.nan)
+    assert raw.ripple_sensitivity_profile(bad, 1, 2, out) == lib.EINVAL
+    assert raw.ripple_sensitivity_profile(bad, 0, 2, out) == lib.EINVAL
+    assert raw.ripple_sensitivity_profile(None, 1, 2, out) == lib.EINVAL
+
+
+def test_profiling_entry_points_reject_before_any_cuda_work(lib):
+    raw = lib._lib
+    fake = 1 << 20  # aligned, never dereferenced: every call below fails validation first
+    d = lib.CacheDesc(1, 2, 64, 128, lib.BF16)
+    for args in [(fake, fake, 0.1, -1, 10, fake), (fake, fake, 0.1, 10, 65, fake),
+                 (fake, fake, 0.1, 20, 10, fake), (fake, fake, -0.5, 0, 10, fake),
+                 (fake, fake, math.inf, 0, 10, fake), (fake, None, 0.1, 0, 10, fake),
+                 (fake + 8, fake, 0.1, 0, 10, fake), (None, fake, 0.1, 0, 10, fake)]:
+        assert raw.ripple_perturb_values(ctypes.byref(d), *args, None) == lib.EINVAL, args
+    for bad in (lib.CacheDesc(1, 2, 64, 96, lib.BF16), lib.CacheDesc(0, 2, 64, 128, lib.BF16),
+                lib.CacheDesc(1, 2, 64, 128, 7)):
+        assert raw.ripple_perturb_values(ctypes.byref(bad), fake, fake, 0.1, 0, 10, fake,
+                                         None) == lib.EINVAL
+    n = lib.ripple_window_kl_workspace_bytes(32, 32, 128256)
+    assert n >= 32 * 32 * 16 * 20 and n % 256 == 0
+    for args in [(0, 4, 64), (2, 0, 64), (2, 4, 12), (2, 4, 0)]:
+        with pytest.raises(lib.RippleError):
+            lib.ripple_window_kl_workspace_bytes(*args)
+    kl = raw.ripple_window_kl
+    assert kl(fake, fake, 2, 4, 64, lib.F32, None, fake, fake, 0, None, None) == lib.EWORKSPACE
+    assert kl(fake, fake, 2, 4, 60, lib.F32, None, fake, fake, 1 << 30, None, None) == lib.EINVAL
+    assert kl(fake, fake, 2, 4, 64, 5, None, fake, fake, 1 << 30, None, None) == lib.EINVAL
+    assert kl(fake, None, 2, 4, 64, lib.F32, None, fake, fake, 1 << 30, None, None) == lib.EINVAL
+    assert kl(fake, fake, 2, 4, 64, lib.F32, None, None, fake, 1 << 30, None, None) == lib.EINVAL
+    assert kl(fake + 4, fake, 2, 4, 64, lib.F32, None, fake, fake, 1 << 30, None, None) == lib.EINVAL
+    assert kl(fake, fake, 2, 4, 64, lib.F32, None, fake, fake + 16, 1 << 30, None, None) == lib.EINVAL
