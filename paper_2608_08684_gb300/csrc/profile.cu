@@ -8,13 +8,14 @@
 //   the squared norm is summed by shuffles among the row's lanes. Each warp
 //   issues the loads of kPerturbUnroll row groups before any arithmetic.
 // kl_stream_kernel: every logits row is cut into slices of kKlSlice entries;
-//   each (set, position, slice) item is reduced to the softmax statistics of
-//   p, (max, sum of exp, P-weighted p - q), and of q, (max, sum of exp). One
-//   CTA per SM takes a contiguous run of items ordered with the set
-//   innermost: a producer lane streams the q slices through a ring of bulk
-//   async (TMA) copies into shared memory, and the consumer warps keep the
-//   shared reference slice p and exp(p - max) in registers across the sets,
-//   so p is read from HBM about once and its exponentials computed once.
+//   each consumer warp reduces its share of every (set, position, slice) item
+//   to the softmax statistics of p, (max, sum of exp, P-weighted p - q), and
+//   of q, (max, sum of exp). One CTA per SM takes a contiguous run of items
+//   ordered with the set innermost: a producer lane streams the q slices
+//   through a ring of bulk async (TMA) copies into shared memory, and the
+//   consumer warps keep the shared reference slice p and exp(p - max) in
+//   registers across the sets, so p is read from HBM about once and its
+//   exponentials computed once.
 //   Each warp writes its own partial per item (no CTA-wide barrier).
 // kl_combine_kernel: one CTA per set, a warp per window position merges the
 //   position's partials, and a fixed-order sum gives the window mean.
@@ -45,7 +46,8 @@ struct KlCfg {
   static constexpr int E = CH * V16;  // 32 logits
 };
 
-// Softmax statistics of one slice, relative to the slice maxima.
+// Softmax statistics of one consumer warp's share of a slice (1024 logits),
+// relative to that share's maxima.
 struct KlPart {
   float mp, zp, ap;  // max p, sum exp(p - mp), sum exp(p - mp) * (p - q)
   float mq, zq;      // max q, sum exp(q - mq)
