@@ -390,12 +390,12 @@ ripple_status ripple_window_kl_workspace_bytes(int32_t n_sets, int32_t n_pos, in
  * d_out      fp32 [n_sets] window averages
  * workspace  device scratch of at least ripple_window_kl_workspace_bytes
  *            bytes, 256-byte aligned, no initialisation needed
- * Each row is cut into fixed slices of 8192 logits; a slice is reduced in
- * fp32 to (max, sum of exponentials, P-weighted logit difference) for p and
- * (max, sum) for q, the slices of a row are merged in a fixed order and the
- * divergence is formed in double, so results do not depend on the GPU or on
- * the run. Identical p and q rows give exactly 0. The call may be captured
- * in a CUDA graph.
+ * Each row is cut into fixed slices of 8192 logits and each slice into fixed
+ * shares of 1024; a share is reduced in fp32 to (max, sum of exponentials,
+ * P-weighted logit difference) for p and (max, sum) for q, the shares of a
+ * row are merged in a fixed order in fp32 and the window mean is summed in
+ * double, so results do not depend on the GPU or on the run. Identical p and
+ * q rows give exactly 0. The call may be captured in a CUDA graph.
  * Errors: RIPPLE_EINVAL (n_sets < 1, n_pos < 1, bad vocab or dtype, NULL or
  * misaligned pointers), RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status:
  * RIPPLE_ETIMEOUT (a bounded in-kernel wait ran out).
