@@ -38,7 +38,9 @@ def _rank_main(rank, world, port, out):
 def test_two_replicas_max_time_and_distinct_batches():
     world = 2
     port = _free_port()
-    with mp.Manager() as m:
+    # the manager's server process is spawned too: forking this
+    # multi-threaded process could deadlock the child
+    with mp.get_context("spawn").Manager() as m:
         out = m.dict()
         mp.spawn(_rank_main, args=(world, port, out), nprocs=world, join=True)
         res = dict(out)
