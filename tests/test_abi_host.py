@@ -171,3 +171,66 @@ def test_profiling_entry_points_reject_before_any_cuda_work(lib):
     assert kl(fake, fake, 2, 4, 64, lib.F32, None, None, fake, 1 << 30, None, None) == lib.EINVAL
     assert kl(fake + 4, fake, 2, 4, 64, lib.F32, None, fake, fake, 1 << 30, None, None) == lib.EINVAL
     assert kl(fake, fake, 2, 4, 64, lib.F32, None, fake, fake + 16, 1 << 30, None, None) == lib.EINVAL
+
+
+def test_compress_and_decode_argument_table(lib):
+    # Every call below is invalid and must be refused on the host, outputs
+    # untouched; none reaches a CUDA call (the fake pointers are never used).
+    raw = lib._lib
+    fake, mis = 1 << 20, (1 << 20) + 8
+    d = lib.layer_desc(1, 4, 2, 128, 512, 32)
+    need = lib.ripple_compress_workspace_bytes(d)
+    base = dict(budget=100, q=fake, k=fake, v=fake, ko=fake, vo=fake, cap=128, idx=fake,
+                scores=None, ws=fake, wsb=need)
+
+    def compress(**over):
+        a = dict(base, **over)
+        n = ctypes.c_int32(-7)
+        st = raw.ripple_compress_layer(ctypes.byref(d), a["budget"], a["q"], a["k"], a["v"],
+                                       a["ko"], a["vo"], a["cap"], a["idx"], a["scores"],
+                                       ctypes.byref(n), a["ws"], a["wsb"], None, None)
+        assert n.value == -7, over
+        return st
+
+    for key in ("q", "k", "v", "ko", "vo", "idx", "ws"):
+        assert compress(**{key: None}) == lib.EINVAL, key
+        assert compress(**{key: mis}) == lib.EINVAL, key
+    assert compress(scores=mis) == lib.EINVAL
+    assert compress(ws=fake + 16) == lib.EINVAL  # workspace must be 256-byte aligned
+    assert compress(budget=-1) == lib.EINVAL
+    assert compress(cap=99) == lib.EINVAL        # n = 100 rows do not fit
+    assert compress(wsb=need - 1) == lib.EWORKSPACE
+    assert raw.ripple_select_layer(ctypes.byref(d), 100, None, fake, fake, fake, fake, 128, fake,
+                                   ctypes.byref(ctypes.c_int32()), fake, need, None,
+                                   None) == lib.EINVAL
+
+    L = 2
+    ptrs = lambda *xs: (ctypes.c_void_p * L)(*xs)
+    caps = (ctypes.c_int32 * L)(16, 16)
+    dd = lib.decode_desc(L, 1, 4, 2, 64)
+    dneed = lib.ripple_decode_workspace_bytes(dd, [16, 16])
+
+    def decode(desc=dd, q=fake, kc=None, vc=None, cp=caps, ws=fake, wsb=dneed):
+        kc = kc if kc is not None else ptrs(fake, fake)
+        vc = vc if vc is not None else ptrs(fake, fake)
+        return raw.ripple_decode_attn(ctypes.byref(desc), q, fake, fake, kc, vc, cp, fake, fake,
+                                      ws, wsb, None, None)
+
+    for bad in (lib.decode_desc(L, 1, 6, 2, 64),          # G = 3
+                lib.decode_desc(L, 1, 32, 2, 64),         # G = 16
+                lib.decode_desc(0, 1, 4, 2, 64),
+                lib.decode_desc(lib.MAX_LAYERS + 1, 1, 4, 2, 64),
+                lib.decode_desc(L, 1, 4, 2, 80),
+                lib.decode_desc(L, 1, 4, 2, 64, scale=-1.0)):
+        assert decode(desc=bad) == lib.EINVAL
+    assert decode(q=None) == lib.EINVAL
+    assert decode(q=mis) == lib.EINVAL
+    assert decode(kc=ptrs(fake, None)) == lib.EINVAL
+    assert decode(vc=ptrs(mis, fake)) == lib.EINVAL
+    assert decode(cp=(ctypes.c_int32 * L)(16, 0)) == lib.EINVAL
+    assert decode(ws=None) == lib.EINVAL
+    assert decode(ws=fake + 16) == lib.EINVAL
+    assert decode(wsb=dneed - 1) == lib.EWORKSPACE
+    assert raw.ripple_decode_attn_noalloc(ctypes.byref(lib.decode_desc(L, 1, 6, 2, 64)), fake,
+                                          fake, fake, ptrs(fake, fake), ptrs(fake, fake), caps,
+                                          fake, fake, None, None) == lib.EINVAL
