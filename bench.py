@@ -18,6 +18,11 @@ against the measured HBM copy bandwidth.
 
 --impl reference times the CPU oracle (the test-infrastructure restatement of
 the paper) on a bounded sample of the same workload, extrapolated to a step.
+
+--case compress|decode times one entry point of the serving path alone;
+--case perturb|kl times the offline profiling kernels (Sec. 4.3: Eq. 6 on one
+layer's V cache, Eq. 7 for one perturbed run per layer); each prints one JSON
+line with its algorithmic bytes and fraction of the measured HBM bandwidth.
 """
 from __future__ import annotations
 
