@@ -49,7 +49,8 @@ typedef enum {
   RIPPLE_EFULL = 3,      /* decode: a layer's cache had no free row to append */
   RIPPLE_ECUDA = 4,      /* a CUDA runtime call failed (launch, attribute, ...) */
   RIPPLE_ETIMEOUT = 5,   /* a bounded in-kernel wait ran out (device status) */
-  RIPPLE_EBOUNDS = 6     /* a kernel met an out-of-range index (device status) */
+  RIPPLE_EBOUNDS = 6,    /* a kernel met an out-of-range index (device status) */
+  RIPPLE_ENOMEM = 7      /* a host-side allocation failed */
 } ripple_status;
 
 typedef enum { RIPPLE_F32 = 0, RIPPLE_BF16 = 1 } ripple_dtype;
@@ -90,7 +91,8 @@ typedef enum {
  * global_budget  B >= 0, tokens summed over layers (per sequence and KV head).
  * budgets_host   [n_layers] output b_l.
  * Returns RIPPLE_EINVAL for NULL pointers, n_layers < 1, ratio < 1 or not
- * finite, 0 < gamma < 1, NaN gamma, a non-finite s_l or global_budget < 0.
+ * finite, 0 < gamma < 1, NaN gamma, a non-finite s_l or global_budget < 0;
+ * RIPPLE_ENOMEM if its host scratch (16 bytes per layer) cannot be allocated.
  * Pure, reentrant, no CUDA calls.
  */
 ripple_status ripple_alloc_budgets(const double *sens_host, int32_t n_layers, double ratio,
@@ -260,17 +262,21 @@ ripple_status ripple_decode_workspace_bytes(const ripple_decode_desc *desc,
  * lens         device int32 [L]: rows in use per layer (same for every b, h);
  *              read, then incremented by one per layer
  * out          device fp32 [L][B][Hq][d]
- * workspace    device scratch of at least ripple_decode_workspace_bytes bytes.
- *              Its leading block holds the step's work counters. Every call
- *              leaves that block at zero, and the library clears it only when
- *              the workspace differs from the one its previous call on the
- *              device used; so between consecutive calls with the same
- *              workspace the caller must not write into it (another buffer
- *              is fine). After a call that ended with RIPPLE_ETIMEOUT in
- *              *dev_status, pass a different workspace or zero the block.
+ * workspace    device scratch of at least ripple_decode_workspace_bytes bytes,
+ *              256-byte aligned. Its contents need no initialisation and may
+ *              be anything between calls (memory freed and handed out again
+ *              by an allocator included): the kernel's first thread block
+ *              zeroes the step's work counters at the start of every call
+ *              and the other blocks touch no counter before it has done so.
+ *              Calls that share a workspace must be ordered on the GPU (same
+ *              stream, or events).
  * Consecutive calls on one stream may overlap: a call's thread blocks may
  * start while the previous call's last blocks finish; they read nothing the
  * previous call writes before it has completed.
+ * After a call that reported RIPPLE_ETIMEOUT its outputs, appended rows and
+ * lengths are unspecified; later calls are unaffected (a CUDA graph holding
+ * that call should be captured again, since its replays reuse the call's
+ * counter tag).
  * The call may be captured in a CUDA graph (no host synchronisation, no
  * allocation); capture was tested after one call outside the capture.
  * A layer with lens[l] >= caps_host[l] (or lens[l] < 0) is not appended to,
@@ -307,14 +313,12 @@ ripple_status ripple_decode_attn(const ripple_decode_desc *desc, const void *q,
  * - Returns RIPPLE_EWORKSPACE, before enqueuing anything, when the step needs
  *   more scratch than the array holds (ripple_decode_workspace_bytes(desc,
  *   caps) > RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES).
- * - Every call on a device shares the one array. Its counters start at zero
- *   (the array is zero-initialised when the library is loaded) and every call
- *   leaves them at zero (the kernel resets them as it exits); every partial
- *   a call reads it has rewritten, so nothing carries over from the previous
- *   call. A call that ended with RIPPLE_ETIMEOUT may leave the counters
- *   dirty: later calls of this entry point on that device are then invalid.
- *   Calls that may overlap on the GPU (different streams without ordering)
- *   race on it; order them, e.g. by issuing them on one stream.
+ * - Every call on a device shares the one array. Each call zeroes the
+ *   counters it uses before using them, and every partial a call reads it
+ *   has written itself, so nothing carries over from the previous call (not
+ *   even from one that reported RIPPLE_ETIMEOUT). Calls that may overlap on
+ *   the GPU (different streams without ordering) race on it; order them,
+ *   e.g. by issuing them on one stream.
  */
 #define RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES (8u << 20)
 ripple_status ripple_decode_attn_noalloc(const ripple_decode_desc *desc, const void *q,
@@ -421,6 +425,20 @@ ripple_status ripple_sensitivity_profile(const double *d_host, int32_t n_example
 /* Number of kernels this library has launched in this process so far
  * (host-side count of launch calls; for benchmarks and launch accounting). */
 uint64_t ripple_kernel_launches(void);
+
+/*
+ * ripple_set_wait_limit_cycles -- bound of the in-kernel waits of kernels
+ * launched from now on, in SM clock cycles (process-wide; returns the
+ * previous value). cycles <= 0 restores the default, 4e9 cycles (about two
+ * seconds). Every wait of a thread block on another role, on another thread
+ * block or on its own bulk copies gives up after this many cycles, reports
+ * RIPPLE_ETIMEOUT in *dev_status and lets the kernel leave; the waits that
+ * then hold a block until the copies it issued have landed keep the default
+ * bound. A diagnostic and test hook (a small limit makes the waits give up
+ * on purpose); the paper has no counterpart. Launches already enqueued keep
+ * the limit they were given.
+ */
+int64_t ripple_set_wait_limit_cycles(int64_t cycles);
 
 /* Human-readable name of a status code (static string). */
 const char *ripple_status_string(int32_t status);

@@ -4,7 +4,6 @@ Submodules:
   ripple  -- ctypes binding of the C-ABI library libripple.so (the product path)
   synth   -- seeded synthetic inputs (no step of the method)
   build   -- in-tree build of libripple.so with nvcc/gcc
-  replica -- host logic of independent multi-GPU replicas
 
 Nothing is imported eagerly, so that importing the package never loads CUDA.
 """

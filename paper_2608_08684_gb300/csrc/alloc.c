@@ -39,7 +39,7 @@ ripple_status ripple_alloc_budgets(const double *sens_host, int32_t n_layers, do
 
   const int n = n_layers;
   double *w = (double *)malloc(sizeof(double) * (size_t)n * 2);
-  if (w == NULL) return RIPPLE_EINVAL;
+  if (w == NULL) return RIPPLE_ENOMEM;
   double *frac = w + n;
 
   /* Eq. 9: min-max normalisation; identical sensitivities give s_hat = 0. */
@@ -111,6 +111,7 @@ const char *ripple_status_string(int32_t status) {
     case RIPPLE_ECUDA: return "CUDA error";
     case RIPPLE_ETIMEOUT: return "in-kernel wait timed out";
     case RIPPLE_EBOUNDS: return "index out of range";
+    case RIPPLE_ENOMEM: return "host allocation failed";
     default: return "unknown status";
   }
 }

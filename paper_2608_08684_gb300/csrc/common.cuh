@@ -12,6 +12,12 @@ namespace ripple {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Default bound of an in-kernel wait: ~2 s at the SM clock. The waits that
+// hold a thread block until its own bulk copies have landed (after another
+// wait gave up) always use this bound; the others use the limit the kernel is
+// launched with (ripple_set_wait_limit_cycles, default this value).
+constexpr long long kDefaultWaitCycles = 4000000000LL;
+
 // ---------------------------------------------------------------- elements
 
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -70,6 +76,16 @@ __device__ __forceinline__ void report(int32_t *status, int32_t code) {
 
 // ---------------------------------------------------------------- PTX wrappers
 
+// GPU-scope acquire load / release store of a flag in global memory.
+__device__ __forceinline__ int ld_acquire(const int *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(int *p, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
@@ -120,7 +136,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 // cycles (about two seconds by default), then reports RIPPLE_ETIMEOUT and
 // returns false instead of hanging.
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, int32_t *status,
-                                          long long max_cycles = 4000000000LL) {
+                                          long long max_cycles = kDefaultWaitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {

@@ -19,6 +19,9 @@ static size_t round_up(size_t x) { return (x + 255) & ~(size_t)255; }
 static std::atomic<uint64_t> g_launches{0};
 void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 
+static std::atomic<long long> g_wait_limit{kDefaultWaitCycles};
+long long wait_limit_cycles() { return g_wait_limit.load(std::memory_order_relaxed); }
+
 CompressWs carve_compress_ws(const LayerGeom &g, void *base) {
   CompressWs w{};
   uint8_t *p = (uint8_t *)base;
@@ -77,6 +80,11 @@ static bool make_geom(const ripple_layer_desc *d, LayerGeom *g) {
 using namespace ripple;
 
 extern "C" uint64_t ripple_kernel_launches(void) { return g_launches.load(); }
+
+extern "C" int64_t ripple_set_wait_limit_cycles(int64_t cycles) {
+  const long long v = cycles > 0 ? (long long)cycles : kDefaultWaitCycles;
+  return (int64_t)g_wait_limit.exchange(v);
+}
 
 extern "C" ripple_status ripple_compress_workspace_bytes(const ripple_layer_desc *desc,
                                                          size_t *bytes_host) {

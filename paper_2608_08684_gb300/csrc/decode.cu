@@ -32,16 +32,21 @@
 // group's last finishing item (atomic count) combines the partials in item
 // order (deterministic).
 //
-// Counters are left at zero by the kernel itself (the group combiner and the
-// last CTA to leave reset them), and each launch is a programmatic dependent
-// of the previous one on the stream: its CTAs take SMs as the previous step's
-// CTAs leave and wait (griddepcontrol.wait) until that step has completed.
+// The step's counters live in the caller's workspace, whose contents are
+// arbitrary: CTA 0 zeroes them at the start of every call and then raises an
+// init flag tagged with the call's epoch; the other CTAs use no counter
+// before they see it (their first item needs none). Each launch is a
+// programmatic dependent of the previous one on the stream: its CTAs take
+// SMs as the previous step's CTAs leave and wait (griddepcontrol.wait) until
+// that step has completed.
 // CTA b's first item is item b, so that before that wait it can already
 // prefetch its first sub-chunks into L2.
 // Every wait is bounded; on timeout the CTA raises RIPPLE_ETIMEOUT and all
 // roles leave their loops together.
 #include <math.h>
 
+#include <atomic>
+#include <chrono>
 #include <mutex>
 
 #include "common.cuh"
@@ -63,7 +68,6 @@ constexpr int kMaxStages = 6;
 constexpr float kRescaleLog2 = 8.f;
 constexpr int kSmemBudget = 226 * 1024;
 constexpr int kMiscBytes = 4096;              // barriers, work list, merge statistics
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at the SM clock
 constexpr unsigned kFull = 0xffffffffu;
 
 constexpr int cmax(int a, int b) { return a > b ? a : b; }
@@ -114,6 +118,7 @@ struct DecSmem {
   int base[RIPPLE_MAX_LAYERS + 1];
   int abort_flag;
   int last;
+  int init_seen;  // this CTA has seen the init flag (consumer thread 0's view)
 };
 
 struct ItemInfo {
@@ -146,20 +151,37 @@ __device__ __forceinline__ ItemInfo item_info(const DecParams &p, const S &s, in
 }
 
 // Bounded wait on an mbarrier phase. Gives up when another role of the CTA
-// has given up, or after ~kWaitCycles (then raises the CTA's abort flag and
+// has given up, or after p.wait_cycles (then raises the CTA's abort flag and
 // reports RIPPLE_ETIMEOUT).
 __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, int *abort_flag,
-                                         int32_t *status) {
+                                         const DecParams &p) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*(volatile int *)abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > p.wait_cycles) {
       *(volatile int *)abort_flag = 1;
-      report(status, RIPPLE_ETIMEOUT);
+      report(p.status, RIPPLE_ETIMEOUT);
       return false;
     }
+  }
+}
+
+// Waits until CTA 0 has zeroed this call's counters (the init flag holds the
+// call's epoch). Bounded like wait_bar.
+__device__ __forceinline__ bool wait_init(const DecParams &p, int *abort_flag) {
+  if (ld_acquire(&p.ctrl[kCtrlFlag]) == p.epoch) return true;
+  const long long t0 = clock64();
+  for (;;) {
+    if (ld_acquire(&p.ctrl[kCtrlFlag]) == p.epoch) return true;
+    if (*(volatile int *)abort_flag) return false;
+    if (clock64() - t0 > p.wait_cycles) {
+      *(volatile int *)abort_flag = 1;
+      report(p.status, RIPPLE_ETIMEOUT);
+      return false;
+    }
+    __nanosleep(32);
   }
 }
 
@@ -237,22 +259,50 @@ __device__ __forceinline__ void all_gather(float x, float (&o)[G]) {
 }
 
 // ------------------------------------------------------------ producer
+// Holds the producer until the bulk copies it has issued have landed (the
+// last phase armed on each stage and item slot), so that no copy writes into
+// shared memory after the CTA has left even when the consumers gave up early;
+// when they did not, these phases have long completed. Fixed bound,
+// independent of the launch's wait limit.
+template <typename Tin, int D, int G>
+__device__ __forceinline__ void drain(DecSmem<Tin, D, G> &s, uint32_t j,
+                                      const int (&last_use)[kItemSlots]) {
+  using C = DecCfg<Tin, D, G>;
+  for (uint32_t jj = j > (uint32_t)C::STAGES ? j - C::STAGES : 0; jj < j; ++jj)
+    mbar_wait(&s.full[jj % C::STAGES], (jj / C::STAGES) & 1, nullptr);
+  for (int slot = 0; slot < kItemSlots; ++slot)
+    if (last_use[slot] >= 0)
+      mbar_wait(&s.item_full[slot], (last_use[slot] / kItemSlots) & 1, nullptr);
+}
+
 template <typename Tin, int D, int G>
 __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &s, int total) {
   using C = DecCfg<Tin, D, G>;
   const int units = p.B * p.Hkv;
-  uint32_t j = 0;
-  // The first item of CTA b is item b; later ones come from the counter.
+  uint32_t j = 0;                                // sub-chunk stages armed
+  int last_use[kItemSlots] = {-1, -1, -1, -1};   // last item count that armed each slot
+  static_assert(kItemSlots == 4, "last_use initialiser");
+  // The item after `cur`, fetched from the counter once CTA 0 has zeroed it.
+  auto next_of = [&](int cur) {
+    if (cur >= total || !wait_init(p, &s.abort_flag)) return total;
+    return atomicAdd(&p.ctrl[kCtrlItem], 1) + (int)gridDim.x;
+  };
+  // The first item of CTA b is item b; later ones come from the counter, one
+  // item ahead (for the first item, once its first loads are issued).
   int it = min((int)blockIdx.x, total);
   for (int icount = 0;; ++icount) {
     const int slot = icount % kItemSlots;
-    const int nxt = it < total ? atomicAdd(&p.ctrl[0], 1) + (int)gridDim.x : total;
-    if (!wait_bar(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, &s.abort_flag, p.status))
+    int nxt = icount > 0 ? next_of(it) : -1;
+    if (!wait_bar(&s.item_empty[slot], ((icount / kItemSlots) & 1) ^ 1, &s.abort_flag, p)) {
+      drain(s, j, last_use);
       return;
+    }
     const int cur = min(it, total);
     s.item_id[slot] = cur;
+    last_use[slot] = icount;
     if (cur >= total) {
       mbar_arrive(&s.item_full[slot]);
+      drain(s, j, last_use);  // returns at once unless the consumers gave up
       return;
     }
     const ItemInfo f = item_info(p, s, cur);
@@ -268,8 +318,11 @@ __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &
       const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * C::ROW_BYTES;
       for (int sub = 0; sub < nsub; ++sub, ++j) {
         const int stage = j % C::STAGES;
-        if (!wait_bar(&s.empty[stage], ((j / C::STAGES) & 1) ^ 1, &s.abort_flag, p.status))
+        if (sub == 1 && nxt < 0) nxt = next_of(it);
+        if (!wait_bar(&s.empty[stage], ((j / C::STAGES) & 1) ^ 1, &s.abort_flag, p)) {
+          drain(s, j, last_use);
           return;
+        }
         const int rs = f.r0 + sub * C::CR;
         const int re = min(rs + C::CR, f.len);  // rows >= len are not in the cache yet
         const int nk = re > rs ? re - rs : 0;
@@ -291,6 +344,7 @@ __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &
         }
       }
     }
+    if (nxt < 0) nxt = next_of(it);
     it = nxt;
   }
 }
@@ -310,7 +364,7 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
   uint32_t j = 0;
   for (int icount = 0;; ++icount) {
     const int slot = icount % kItemSlots;
-    bool ok = wait_bar(&s.item_full[slot], (icount / kItemSlots) & 1, &s.abort_flag, p.status);
+    bool ok = wait_bar(&s.item_full[slot], (icount / kItemSlots) & 1, &s.abort_flag, p);
     ok = __all_sync(kFull, ok);
     const int it = ok ? s.item_id[slot] : total;
     // Queries to fp32, scaled to log2 units, in the order the lanes read them:
@@ -436,7 +490,7 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
     const int nsub = (f.rows + C::CR - 1) / C::CR;
     for (int sub = 0; sub < nsub; ++sub, ++j) {
       const int stage = j % C::STAGES;
-      wait_bar(&s.full[stage], (j / C::STAGES) & 1, &s.abort_flag, p.status);
+      wait_bar(&s.full[stage], (j / C::STAGES) & 1, &s.abort_flag, p);
       __syncwarp();
       const int nrows = min(C::CR, f.rows - sub * C::CR);
       const Tin *ks = (const Tin *)s.kv[stage][0];
@@ -527,11 +581,14 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
     if (!single) {
       __threadfence();
       named_bar_sync(1, kWarps * 32);
-      if (tid == 0) s.last = atomicAdd(&p.ctrl[2 + f.group], 1) == f.nch - 1;
+      if (tid == 0) {
+        if (!s.init_seen) s.init_seen = wait_init(p, &s.abort_flag);
+        // without the counters (a wait gave up) no item combines the group
+        s.last = s.init_seen && atomicAdd(&p.ctrl[kCtrlGroup + f.group], 1) == f.nch - 1;
+      }
       named_bar_sync(1, kWarps * 32);
       if (s.last) {
         __threadfence();
-        if (tid == 0) p.ctrl[2 + f.group] = 0;  // left at zero for the next call
         for (int e = tid; e < G * D; e += kWarps * 32) {
           const int g = e / D;
           float M = -INFINITY;
@@ -617,9 +674,20 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
       mbar_init(&s.item_empty[i], kWarps);
     }
     s.abort_flag = 0;
+    s.init_seen = 0;
     fence_mbar_init();
   }
+  // CTA 0 zeroes this call's counters (the workspace may hold anything),
+  // then raises the init flag; the other CTAs use no counter before they see
+  // it (wait_init).
+  const int n_ctrl = (kCtrlGroup - kCtrlItem) + p.L * units;
+  if (blockIdx.x == 0)
+    for (int i = tid; i < n_ctrl; i += kThreads) p.ctrl[kCtrlItem + i] = 0;
   __syncthreads();
+  if (blockIdx.x == 0 && tid == 0) {
+    __threadfence();
+    st_release(&p.ctrl[kCtrlFlag], p.epoch);
+  }
   if (tid == 0) {
     int acc = 0;
     for (int t = 0; t < p.L; ++t) {
@@ -638,16 +706,19 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
   }
 
   // The last CTA to leave advances the lengths of the layers it appended to
-  // and leaves the item and exit counters at zero for the next call.
+  // and lowers the init flag (a replay of this launch starts from CTA 0's
+  // zeroing again). A CTA that never saw the flag (its wait gave up) leaves
+  // the counters alone; the call has then reported RIPPLE_ETIMEOUT.
   __syncwarp();
   __syncthreads();
   if (tid == 0) {
+    if (!s.init_seen) s.init_seen = wait_init(p, &s.abort_flag);
     __threadfence();
-    if (atomicAdd(&p.ctrl[1], 1) == (int)gridDim.x - 1) {
+    if (s.init_seen && atomicAdd(&p.ctrl[kCtrlExit], 1) == (int)gridDim.x - 1) {
       for (int t = 0; t < p.L; ++t)
         if (s.len[t] >= 0) p.lens[p.order[t]] = s.len[t] + 1;
-      p.ctrl[0] = 0;
-      p.ctrl[1] = 0;
+      __threadfence();
+      st_release(&p.ctrl[kCtrlFlag], 0);
     }
   }
 }
@@ -656,27 +727,31 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
 
 constexpr int kMaxDevices = 64;
 
+// Per-device caches of the SM count and of the kernels' shared-memory
+// attribute; atomics, as several host threads may make their first calls at
+// once (a repeated look-up or attribute set is harmless).
 int sm_count(int dev) {
-  static int n[kMaxDevices] = {};
+  static std::atomic<int> n[kMaxDevices];
   if (dev < 0 || dev >= kMaxDevices) return 1;
-  if (n[dev] == 0) {
-    int v = 0;
+  int v = n[dev].load(std::memory_order_relaxed);
+  if (v == 0) {
     cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
-    n[dev] = v > 0 ? v : 1;
+    v = v > 0 ? v : 1;
+    n[dev].store(v, std::memory_order_relaxed);
   }
-  return n[dev];
+  return v;
 }
 
 template <typename Tin, int D, int G>
 cudaError_t launch_g(const DecParams &p, int dev, cudaStream_t st) {
-  static bool attr_set[kMaxDevices] = {};
+  static std::atomic<bool> attr_set[kMaxDevices];
   const int smem = (int)sizeof(DecSmem<Tin, D, G>);
   static_assert(sizeof(DecSmem<Tin, D, G>) <= 227 * 1024, "shared memory per CTA");
-  if (!attr_set[dev]) {
+  if (!attr_set[dev].load(std::memory_order_acquire)) {
     const cudaError_t e = cudaFuncSetAttribute(decode_kernel<Tin, D, G>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    attr_set[dev] = true;
+    attr_set[dev].store(true, std::memory_order_release);
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(sm_count(dev));
@@ -704,26 +779,19 @@ cudaError_t launch_d(const DecParams &p, int dev, cudaStream_t st) {
   }
 }
 
-// Counter blocks left at zero by the previous call on each device: the kernel
-// resets its counters as it exits, so a workspace used by the previous call
-// on the device needs no clearing.
-struct CleanCtrl {
-  const void *ptr = nullptr;
-  size_t bytes = 0;
-};
-CleanCtrl g_clean[kMaxDevices];
-std::mutex g_clean_mu;
-
-cudaError_t clear_ctrl_if_needed(int dev, int *ctrl, size_t bytes, cudaStream_t st) {
-  std::lock_guard<std::mutex> lock(g_clean_mu);
-  CleanCtrl &c = g_clean[dev];
-  if (c.ptr == ctrl && c.bytes >= bytes) return cudaSuccess;
-  const cudaError_t e = cudaMemsetAsync(ctrl, 0, bytes, st);
-  if (e == cudaSuccess) {
-    c.ptr = ctrl;
-    c.bytes = bytes;
-  }
-  return e;
+// Epoch of a call: a per-process sequence (never 0) that starts at a value
+// taken from the clock, so that an init flag left in reused memory by an
+// earlier call or process is unlikely to match.
+int next_epoch() {
+  static std::atomic<uint32_t> seq{(uint32_t)std::chrono::steady_clock::now()
+                                       .time_since_epoch()
+                                       .count() *
+                                   2654435761u};
+  uint32_t e;
+  do {
+    e = seq.fetch_add(1, std::memory_order_relaxed) + 1;
+  } while (e == 0);
+  return (int)e;
 }
 
 // Cache rows per work item (the workspace holds one partial per item).
@@ -740,7 +808,7 @@ size_t plan(const ripple_decode_desc *d, const int32_t *caps, void *ws, DecParam
   for (int l = 0; l < d->n_layers; ++l)
     items += (size_t)d->batch * d->n_kv_heads * ((caps[l] + rows - 1) / rows);
   const size_t groups = (size_t)d->n_layers * d->batch * d->n_kv_heads;
-  const size_t ctrl = round_up(sizeof(int) * (2 + groups));
+  const size_t ctrl = round_up(sizeof(int) * (kCtrlGroup + groups));
   const size_t ml = round_up(sizeof(float2) * items * G);
   const size_t o = round_up(sizeof(float) * items * G * d->head_dim);
   if (p != nullptr) {
@@ -750,10 +818,6 @@ size_t plan(const ripple_decode_desc *d, const int32_t *caps, void *ws, DecParam
     p->ws_o = (float *)(base + ctrl + ml);
   }
   return ctrl + ml + o;
-}
-
-size_t ctrl_bytes(const ripple_decode_desc *d) {
-  return sizeof(int) * (2 + (size_t)d->n_layers * d->batch * d->n_kv_heads);
 }
 
 bool desc_ok(const ripple_decode_desc *d) {
@@ -815,11 +879,12 @@ ripple_status prepare(const ripple_decode_desc *desc, const void *q, const void 
   return RIPPLE_OK;
 }
 
-ripple_status run(const ripple_decode_desc *desc, const DecParams &p, void *stream) {
+ripple_status run(const ripple_decode_desc *desc, DecParams &p, void *stream) {
+  p.epoch = next_epoch();
+  p.wait_cycles = wait_limit_cycles();
   cudaStream_t st = (cudaStream_t)stream;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RIPPLE_ECUDA;
-  if (clear_ctrl_if_needed(dev, p.ctrl, ctrl_bytes(desc), st) != cudaSuccess) return RIPPLE_ECUDA;
   cudaError_t e;
   if (desc->dtype == RIPPLE_F32)
     e = desc->head_dim == 64 ? launch_d<float, 64>(p, dev, st) : launch_d<float, 128>(p, dev, st);
@@ -868,11 +933,11 @@ extern "C" ripple_status ripple_decode_attn(const ripple_decode_desc *desc, cons
 // have no way to hand this library a scratch buffer. For those callers the
 // step's control counters and split-K partials live in the file-scope device
 // array below instead of a caller workspace. Every GPU that loads the library
-// keeps it until the process exits; all calls on a device share it. Its
-// counters start at zero (zero-initialised at load) and every call leaves them
-// at zero (the kernel resets them as it exits); every partial a call reads it has
-// rewritten, so no state carries over from the previous call. Calls that
-// overlap on the GPU race on it.
+// keeps it until the process exits; all calls on a device share it. Every
+// call zeroes the counters it uses before using them, and every partial a call
+// reads it has written itself, so no state carries over from the previous call
+// (not even from one that ended with RIPPLE_ETIMEOUT). Calls that overlap on
+// the GPU race on it.
 
 static __device__ __align__(256) float
     g_decode_scratch[RIPPLE_DECODE_NOALLOC_SCRATCH_BYTES / sizeof(float)];

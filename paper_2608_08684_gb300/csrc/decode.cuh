@@ -17,8 +17,11 @@ struct DecParams {
   float *out;
   float *ws_o;      // [items][G][D] unnormalised partial outputs
   float2 *ws_ml;    // [items][G] (max, sum) of each partial
-  int *ctrl;        // [0] item counter, [1] exit counter, [2 + group] items done
+  int *ctrl;        // counters of the step (kCtrl* below)
   int32_t *status;
+  int epoch;        // nonzero tag of this call: the init flag's value once the
+                    // counters are zeroed
+  long long wait_cycles;  // bound of the in-kernel waits
   const void *kc[RIPPLE_MAX_LAYERS];
   const void *vc[RIPPLE_MAX_LAYERS];
   int cap[RIPPLE_MAX_LAYERS];
@@ -26,5 +29,16 @@ struct DecParams {
 };
 
 constexpr int kItemRows = 4096;  // cache rows per work item
+
+// Control block of a step in the workspace (int32 words). The init flag has a
+// 128-byte line to itself; CTA 0 zeroes the counters at the start of every
+// call and then sets the flag to the call's epoch, and the other CTAs use no
+// counter before they have seen it. The last CTA to leave sets the flag back
+// to 0, so that a replay of the same launch (same epoch) waits for CTA 0
+// again.
+constexpr int kCtrlFlag = 0;    // init flag
+constexpr int kCtrlItem = 32;   // work-item counter
+constexpr int kCtrlExit = 33;   // CTAs that have left
+constexpr int kCtrlGroup = 34;  // + group: items of the group finished
 
 }  // namespace ripple

@@ -31,7 +31,8 @@ struct GatherTable {
 
 __global__ void __launch_bounds__(kThreads) gather_kernel(const __grid_constant__ GatherTable tab,
                                                           int T, int row_bytes,
-                                                          int32_t *status) {
+                                                          int32_t *status,
+                                                          long long wait_cycles) {
   extern __shared__ __align__(128) uint8_t tile[];
   __shared__ __align__(8) uint64_t bar;
   const int layer = blockIdx.y / tab.upl, unit = blockIdx.y % tab.upl;
@@ -64,7 +65,10 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const __grid_constant_
     bulk_g2s(tk + (size_t)r * row_bytes, k + (unit_in + t) * row_bytes, row_bytes, &bar);
     bulk_g2s(tv + (size_t)r * row_bytes, v + (unit_in + t) * row_bytes, row_bytes, &bar);
   }
-  const bool ok = mbar_wait(&bar, 0, status);
+  const bool ok = mbar_wait(&bar, 0, status, wait_cycles);
+  // After a wait that gave up, hold the block until its copies have landed
+  // (fixed bound), so that none writes into shared memory after it has left.
+  if (!ok) mbar_wait(&bar, 0, nullptr);
   __syncthreads();
   if (bad) report(status, RIPPLE_EBOUNDS);
   if (threadIdx.x == 0 && ok) {
@@ -105,7 +109,7 @@ cudaError_t launch_gather(const LayerGeom &g, int n_layers, const void *const *k
                                        (int)smem);
   if (e != cudaSuccess) return e;
   const dim3 grid((max_keep + kTileRows - 1) / kTileRows, g.units * n_layers);
-  gather_kernel<<<grid, kThreads, smem, st>>>(tab, g.T, row_bytes, status);
+  gather_kernel<<<grid, kThreads, smem, st>>>(tab, g.T, row_bytes, status, wait_limit_cycles());
   count_launches(1);
   return cudaGetLastError();
 }

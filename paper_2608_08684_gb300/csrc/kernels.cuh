@@ -12,6 +12,10 @@ namespace ripple {
 // Host-side count of kernel launches (ripple_kernel_launches).
 void count_launches(int n);
 
+// Bound, in SM clock cycles, that kernels launched now give their in-kernel
+// waits (ripple_set_wait_limit_cycles; kDefaultWaitCycles unless changed).
+long long wait_limit_cycles();
+
 // Geometry of one layer's compression, derived from ripple_layer_desc.
 struct LayerGeom {
   int B, Hq, Hkv, G, D, T, W, P, R;  // R = G * W window rows per unit

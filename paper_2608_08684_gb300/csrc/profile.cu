@@ -36,7 +36,6 @@ constexpr int kKlSlice = 8192;                           // logits per work item
 constexpr int kKlStageBytes = kKlSlice * 4;              // a fp32 slice
 constexpr int kKlStages = 4;                             // q ring: 128 KB in flight
 constexpr int kKlCombineThreads = 1024;
-constexpr long long kKlWaitCycles = 4000000000LL;        // ~2 s at the SM clock
 
 // A consumer thread's share of a slice: CH chunks of V16 logits (16 bytes).
 template <typename Tl>
@@ -178,15 +177,15 @@ __device__ __forceinline__ float warp_sum_rn(float v) {
 }
 
 // Bounded mbarrier wait; gives up when another role has given up, or after
-// ~kKlWaitCycles (then raises the abort flag and reports RIPPLE_ETIMEOUT).
+// `limit` cycles (then raises the abort flag and reports RIPPLE_ETIMEOUT).
 __device__ __forceinline__ bool kl_wait(uint64_t *bar, uint32_t parity, int *abort_flag,
-                                        int32_t *status) {
+                                        int32_t *status, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*(volatile int *)abort_flag) return false;
-    if (clock64() - t0 > kKlWaitCycles) {
+    if (clock64() - t0 > limit) {
       *(volatile int *)abort_flag = 1;
       report(status, RIPPLE_ETIMEOUT);
       return false;
@@ -274,7 +273,8 @@ __device__ __forceinline__ void share_stats(const float (&x)[KlCfg<Tl>::E],
 template <typename Tl>
 __global__ void __launch_bounds__(kKlThreads, 1)
     kl_stream_kernel(const Tl *__restrict__ p, const Tl *__restrict__ q, int n_sets, int n_pos,
-                     int vocab, int n_slices, long long n_items, KlPart *part, int32_t *status) {
+                     int vocab, int n_slices, long long n_items, KlPart *part, int32_t *status,
+                     long long wait_cycles) {
   using C = KlCfg<Tl>;
   extern __shared__ __align__(128) uint8_t smem_raw[];
   KlSmem &s = *reinterpret_cast<KlSmem *>(smem_raw);
@@ -307,13 +307,13 @@ __global__ void __launch_bounds__(kKlThreads, 1)
       const uint32_t bytes = (uint32_t)(min(kKlSlice, vocab - begin) * (int)sizeof(Tl));
       if (item == i0 || set == 0) {
         const int ps = pc & 1;
-        if (!kl_wait(&s.p_empty[ps], ((pc >> 1) & 1) ^ 1, &s.abort_flag, status)) break;
+        if (!kl_wait(&s.p_empty[ps], ((pc >> 1) & 1) ^ 1, &s.abort_flag, status, wait_cycles)) break;
         mbar_arrive_expect_tx(&s.p_full[ps], bytes);
         bulk_g2s(s.p[ps], p + (size_t)pos * vocab + begin, bytes, &s.p_full[ps]);
         ++pc;
       }
       const int st = qc % kKlStages;
-      if (!kl_wait(&s.q_empty[st], ((qc / kKlStages) & 1) ^ 1, &s.abort_flag, status)) break;
+      if (!kl_wait(&s.q_empty[st], ((qc / kKlStages) & 1) ^ 1, &s.abort_flag, status, wait_cycles)) break;
       mbar_arrive_expect_tx(&s.q_full[st], bytes);
       bulk_g2s(s.q[st], q + ((size_t)set * n_pos + pos) * vocab + begin, bytes, &s.q_full[st]);
       ++qc;
@@ -322,11 +322,11 @@ __global__ void __launch_bounds__(kKlThreads, 1)
     // otherwise the consumers have already seen every phase complete).
     for (uint32_t j = qc > (uint32_t)kKlStages ? qc - kKlStages : 0; j < qc; ++j) {
       int never = 0;
-      kl_wait(&s.q_full[j % kKlStages], (j / kKlStages) & 1, &never, status);
+      kl_wait(&s.q_full[j % kKlStages], (j / kKlStages) & 1, &never, status, kDefaultWaitCycles);
     }
     for (uint32_t j = pc > 2u ? pc - 2 : 0; j < pc; ++j) {
       int never = 0;
-      kl_wait(&s.p_full[j & 1], (j >> 1) & 1, &never, status);
+      kl_wait(&s.p_full[j & 1], (j >> 1) & 1, &never, status, kDefaultWaitCycles);
     }
     return;
   }
@@ -347,7 +347,7 @@ __global__ void __launch_bounds__(kKlThreads, 1)
     const int len = min(kKlSlice, vocab - slice * kKlSlice);
     if (item == i0 || set == 0) {
       const int ps = pc & 1;
-      if (!__all_sync(0xffffffffu, kl_wait(&s.p_full[ps], (pc >> 1) & 1, &s.abort_flag, status)))
+      if (!__all_sync(0xffffffffu, kl_wait(&s.p_full[ps], (pc >> 1) & 1, &s.abort_flag, status, wait_cycles)))
         break;
       read_share<Tl>(s.p[ps], ctid, len, pv, pok);
       __syncwarp();
@@ -357,7 +357,7 @@ __global__ void __launch_bounds__(kKlThreads, 1)
     }
     const int st = qc % kKlStages;
     if (!__all_sync(0xffffffffu,
-                    kl_wait(&s.q_full[st], (qc / kKlStages) & 1, &s.abort_flag, status)))
+                    kl_wait(&s.q_full[st], (qc / kKlStages) & 1, &s.abort_flag, status, wait_cycles)))
       break;
     float qv[C::E];
     bool qok[C::CH];
@@ -486,7 +486,7 @@ cudaError_t launch_kl(const void *p, const void *q, int n_sets, int n_pos, int v
   if (e != cudaSuccess) return e;
   const int grid = (int)(n_items < sms ? n_items : sms);  // one CTA per SM
   kernel<<<grid, kKlThreads, smem, st>>>((const Tl *)p, (const Tl *)q, n_sets, n_pos, vocab,
-                                         n_slices, n_items, part, status);
+                                         n_slices, n_items, part, status, wait_limit_cycles());
   kl_combine_kernel<<<n_sets, kKlCombineThreads, 0, st>>>(part, n_pos,
                                                           n_slices * kKlConsumerWarps, kl_out,
                                                           d_out);

@@ -47,7 +47,7 @@ constexpr int kTileBytes = 2 * kHalfBytes;      // one 128 x 128 bf16 tile
 constexpr int kThreads = 352;
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 14;
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz
+
 
 // ------------------------------------------------------------ work list
 
@@ -62,6 +62,7 @@ struct TcParams {
   float *votes;     // [units][P]
   int *ctrl;        // [u] items of unit u published; [units + u] row statistics ready
   int32_t *status;
+  long long wait_cycles;  // bound of the in-kernel waits
 };
 
 struct ItemRef {
@@ -107,6 +108,7 @@ struct Misc {
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots];
   uint32_t tmem_base;
   int abort_flag;
+  long long wait_cycles;  // bound of the waits of this launch
   alignas(16) float off[2][256];  // per-warpgroup row log-normalisers of a pass-2 item
   float2 pstat[kPubSlots][2][256];  // pass-1 row statistics per slot and warpgroup
 };
@@ -126,7 +128,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *m
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*(volatile int *)&ms->abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > ms->wait_cycles) {
       *(volatile int *)&ms->abort_flag = 1;
       report(status, RIPPLE_ETIMEOUT);
       return false;
@@ -148,7 +150,7 @@ __device__ __forceinline__ bool wait_ready(const int *flag, Misc *ms, int32_t *s
   for (;;) {
     if (ld_acquire(flag)) return true;
     if (*(volatile int *)&ms->abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > ms->wait_cycles) {
       *(volatile int *)&ms->abort_flag = 1;
       report(status, RIPPLE_ETIMEOUT);
       return false;
@@ -198,6 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&ms->mma_done, 1);
     ms->abort_flag = 0;
+    ms->wait_cycles = p.wait_cycles;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -244,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Let every issued copy land before the CTA can exit (matters only after
       // an abort; in normal operation every stage was already consumed).
       for (int j = max(0, kcount - C::NK); j < kcount; ++j)
-        mbar_wait(&ms->k_full[j % C::NK], (j / C::NK) & 1, nullptr, kWaitCycles / 4);
+        mbar_wait(&ms->k_full[j % C::NK], (j / C::NK) & 1, nullptr);
     } else if (lane == 1) {
       int qcount = 0;
       for (int k = 0; k < n; ++k) {
@@ -262,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++qcount;
       }
       for (int k = max(0, qcount - C::NQ); k < qcount; ++k)
-        mbar_wait(&ms->q_full[k % C::NQ], (k / C::NQ) & 1, nullptr, kWaitCycles / 4);
+        mbar_wait(&ms->q_full[k % C::NQ], (k / C::NQ) & 1, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
@@ -318,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // All issued MMAs complete before TMEM is released.
       mma_commit(&ms->mma_done);
-      mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
+      mbar_wait(&ms->mma_done, 0, nullptr);
     }
   } else if (warp == 10) {
     // ------------------------------------------------ publisher of pass-1 results
@@ -615,6 +618,7 @@ cudaError_t launch_nr(const LayerGeom &g, const void *q_win, const void *k, cons
   p.votes = votes;
   p.ctrl = ws.counters;
   p.status = status;
+  p.wait_cycles = wait_limit_cycles();
   cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * g.units, st);
   if (e != cudaSuccess) return e;
   constexpr int smem = smem_bytes<NR>();

@@ -47,7 +47,6 @@ constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
 constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then query slots
 static_assert(kQCol + kNQ * 64 <= 512, "TMEM columns");
-constexpr long long kWaitCycles = 4000000000LL;
 
 struct Tc1Params {
   int units, upl, T, P, W, Hq, Hkv, G;  // units of all layers, units per layer
@@ -61,6 +60,7 @@ struct Tc1Params {
   float *votes;      // [units][P], layer-major
   int *ctrl;         // [u] items of unit u published; [units + u] row statistics ready
   int32_t *status;
+  long long wait_cycles;  // bound of the in-kernel waits
 };
 
 struct ItemRef {
@@ -133,6 +133,7 @@ struct Misc {
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
   uint32_t tmem_base;
   int abort_flag;
+  long long wait_cycles;  // bound of the waits of this launch
   float2 pstat[kPubSlots][2][128];      // pass-1 row statistics per slot and warpgroup
   alignas(16) float offs[2][128];       // per warpgroup: the pass-2 item's row log-normalisers
 };
@@ -149,7 +150,7 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *m
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*(volatile int *)&ms->abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > ms->wait_cycles) {
       *(volatile int *)&ms->abort_flag = 1;
       report(status, RIPPLE_ETIMEOUT);
       return false;
@@ -169,7 +170,7 @@ __device__ __forceinline__ bool wait_ready(const int *flag, Misc *ms, int32_t *s
   for (;;) {
     if (ld_acquire(flag)) return true;
     if (*(volatile int *)&ms->abort_flag) return false;
-    if (clock64() - t0 > kWaitCycles) {
+    if (clock64() - t0 > ms->wait_cycles) {
       *(volatile int *)&ms->abort_flag = 1;
       report(status, RIPPLE_ETIMEOUT);
       return false;
@@ -226,6 +227,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&ms->mma_done, 1);
     ms->abort_flag = 0;
+    ms->wait_cycles = p.wait_cycles;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -283,8 +285,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       for (int j = max(0, kcount - kNK); j < kcount; ++j)
-        mbar_wait(&ms->k_full[j % kNK], (j / kNK) & 1, nullptr, kWaitCycles / 4);
-      if (qcount > 0) mbar_wait(&ms->qs_full, (qcount - 1) & 1, nullptr, kWaitCycles / 4);
+        mbar_wait(&ms->k_full[j % kNK], (j / kNK) & 1, nullptr);
+      if (qcount > 0) mbar_wait(&ms->qs_full, (qcount - 1) & 1, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
@@ -345,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       mma_commit(&ms->mma_done);
-      mbar_wait(&ms->mma_done, 0, nullptr, kWaitCycles / 4);
+      mbar_wait(&ms->mma_done, 0, nullptr);
     }
   } else if (warp == 10) {
     // ------------------------------------------------ publisher of pass-1 results
@@ -654,6 +656,7 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
   p.votes = votes;
   p.ctrl = ws.counters;
   p.status = status;
+  p.wait_cycles = wait_limit_cycles();
   cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * p.units, st);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(score_tc1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -9,7 +9,6 @@ module fails loudly if the library has not been built.
 from __future__ import annotations
 
 import ctypes
-import math
 import os
 
 import torch
@@ -21,7 +20,7 @@ _lib = ctypes.CDLL(LIB_PATH)
 
 F32, BF16 = 0, 1
 POOL_MAX, POOL_AVG, POOL_NONE = 0, 1, 2
-OK, EINVAL, EWORKSPACE, EFULL, ECUDA, ETIMEOUT, EBOUNDS = range(7)
+OK, EINVAL, EWORKSPACE, EFULL, ECUDA, ETIMEOUT, EBOUNDS, ENOMEM = range(8)
 MAX_LAYERS = 128
 COMPRESS_MAX_LAYERS = 80
 _POOLS = {"max": POOL_MAX, "avg": POOL_AVG, "none": POOL_NONE}
@@ -101,6 +100,8 @@ _lib.ripple_window_kl.restype = _i32
 _lib.ripple_sensitivity_profile.argtypes = [ctypes.POINTER(_f64), _i32, _i32,
                                             ctypes.POINTER(_f64)]
 _lib.ripple_sensitivity_profile.restype = _i32
+_lib.ripple_set_wait_limit_cycles.argtypes = [_i64]
+_lib.ripple_set_wait_limit_cycles.restype = _i64
 _lib.ripple_kernel_launches.argtypes = []
 _lib.ripple_kernel_launches.restype = ctypes.c_uint64
 _lib.ripple_status_string.argtypes = [_i32]
@@ -337,5 +338,7 @@ def ripple_kernel_launches() -> int:
     return int(_lib.ripple_kernel_launches())
 
 
-def default_scale(head_dim: int) -> float:
-    return 1.0 / math.sqrt(head_dim)
+def ripple_set_wait_limit_cycles(cycles: int) -> int:
+    """Bound of the in-kernel waits of later launches (SM cycles; <= 0 restores
+    the default of about two seconds); returns the previous bound."""
+    return int(_lib.ripple_set_wait_limit_cycles(int(cycles)))

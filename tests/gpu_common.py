@@ -11,7 +11,15 @@ from paper_2608_08684_gb300 import synth
 SCORE_RTOL = 1e-3      # votes: relative, fp32 accumulation from bf16/fp32 inputs
 SCORE_ATOL_REL = 1e-9  # absolute floor, relative to the largest vote (underflow guard)
 SELECT_GAP_RTOL = 2e-3  # a set mismatch needs two votes within 2x the score tolerance
-DECODE_ATOL = 2e-2     # decode output, max-abs against the fp64 oracle
+DECODE_ATOL = 2e-2     # decode output, max-abs against the fp64 oracle (acceptance bar)
+# Decode output, max-abs: the kernel's own precision. Inputs are exact in fp32;
+# each lane sums its share of a group's rows (at most a few hundred terms of
+# |p v| <= |v|, |v| < 6) in fp32 and the shares merge through short trees, with
+# exponentials of relative error ~2^-22: a worst case of a few 1e-5, observed
+# ~1e-6. Dropping or repeating one row of an n-row cache moves the output by
+# about 1/n (a few 1e-4 at the lengths tested), so this bound sees it where
+# the acceptance bar does not.
+DECODE_PREC_ATOL = 1e-4
 
 
 def layer_inputs(wl, layer, device):
@@ -98,3 +106,12 @@ def check_compress_unit(wl, out, q_win, k, v, b, h, budget, pool="max", scale=No
         assert list(gidx) == list(range(wl.seq_len))
         return 0, 0
     return selection_mismatch(gidx, ref["idx"], ref["pooled"], n, wl.window)
+
+
+def assert_decode_close(got, ref):
+    """Decode outputs against the oracle: the acceptance bar and the kernel's
+    precision bound."""
+    err = float(np.abs(np.asarray(got, np.float64) - ref).max()) if np.size(ref) else 0.0
+    assert err <= DECODE_ATOL, f"max-abs error {err} above the acceptance bar {DECODE_ATOL}"
+    assert err <= DECODE_PREC_ATOL, f"max-abs error {err} above the kernel precision bound"
+    return err

@@ -1,7 +1,10 @@
 """ripple_compress_layers (several layers of one shape in one call, each with
 its own budget) gives, layer by layer, exactly what ripple_compress_layer
-gives: the same kept counts, indices and gathered rows, bit for bit. The
-single-layer path is checked against the oracle in test_gpu_compress.py."""
+gives: the same kept counts, indices and gathered rows, bit for bit; and the
+full 32-layer call of the 32k workload is checked against the oracle on a
+sample of units of every layer. The single-layer path is checked against the
+oracle in test_gpu_compress.py."""
+import numpy as np
 import pytest
 import torch
 
@@ -69,3 +72,46 @@ def test_layers_call_full_size_four_layers(lib):
                                  wl.global_budget)
     wl4 = wl.replace(n_layers=4)
     _both(lib, wl4, [b[12], b[0], b[20], b[31]], device_gen=DEV)
+
+
+def test_layers_call_full_size_all_layers_against_oracle(lib):
+    # The benchmark's own call: ripple_compress_layers over all 32 layers of the
+    # 32k workload (1024 units in flight in one scoring launch, the
+    # one-CTA-per-unit selection) with the allocator's budgets and inputs
+    # generated on the GPU; the oracle checks three units of every layer:
+    # retained sets agree on >= 99.9% with every difference inside the score
+    # tolerance, gathered rows byte-exact.
+    wl = synth.WORKLOADS["llama8b-32k"]
+    budgets = lib.ripple_alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
+                                       wl.global_budget)
+    L, B, H, d = wl.n_layers, wl.batch, wl.n_kv_heads, wl.head_dim
+    desc = lib.layer_desc(B, wl.n_q_heads, H, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                          wl.torch_dtype)
+    ins = [C.layer_inputs(wl, l, DEV) for l in range(L)]
+    ns = [lib.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    k_out = [torch.zeros(B, H, n + 1, d, dtype=wl.torch_dtype, device=DEV) for n in ns]
+    v_out = [torch.zeros_like(x) for x in k_out]
+    idx = [torch.full((B * H * n,), -1, dtype=torch.int32, device=DEV) for n in ns]
+    tables = lib.CompressTables([x[0] for x in ins], [x[1] for x in ins], [x[2] for x in ins],
+                                k_out, v_out, idx)
+    ws = torch.empty(lib.ripple_compress_layers_workspace_bytes(desc, L), dtype=torch.uint8,
+                     device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    assert lib.ripple_compress_layers(desc, budgets, tables, ws, dev_status=status) == ns
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    agree = total = 0
+    for l in range(L):
+        q, k, v = ins[l]
+        out = {"n": ns[l], "idx": idx[l].view(B, H, ns[l]), "k_out": k_out[l],
+               "v_out": v_out[l], "scores": None}
+        # a fixed seeded sample of three units of this layer
+        rng = np.random.default_rng(1000 + l)
+        units = rng.choice(B * H, size=3, replace=False)
+        for u in units:
+            a, t = C.check_compress_unit(wl, out, q, k, v, int(u) // H, int(u) % H, budgets[l])
+            agree += a
+            total += t
+    assert agree >= 0.999 * total
+    del ins, tables, k_out, v_out, idx, ws
+    torch.cuda.empty_cache()
