@@ -37,7 +37,7 @@ CompressWs carve_compress_ws(const LayerGeom &g, void *base) {
   w.row_lognorm = (float *)take(sizeof(float) * g.units * g.R);
   w.votes = (float *)take(sizeof(float) * g.units * (size_t)g.P);
   w.keys = (uint32_t *)take(g.P > kSelectSmemKeys ? sizeof(uint32_t) * g.units * (size_t)g.P : 0);
-  w.counters = (int32_t *)take(sizeof(int32_t) * (32 + 2 * (size_t)g.units));
+  w.counters = (int32_t *)take(sizeof(int32_t) * (128 + 2 * (size_t)g.units));
   w.bytes = off;
   return w;
 }

@@ -1,28 +1,26 @@
 // Observation-window token scoring for G * w = 128 window rows (SnapKV's rule
 // as RippleKV keeps it, Sec. 4.4, last paragraph), bf16, d = 128, on the
-// 5th-generation tensor cores with the window queries held in TMEM.
+// 5th-generation tensor cores.
 //
-// Same work split as score_tc.cu (one persistent CTA per SM, item i on CTA
-// i mod grid, each CTA running P1(a_k) then P2(a_k-1) in its step k so that
-// keys are re-read from L2 one item after their first read, a publisher warp
-// merging pass-1 row statistics). Each pass takes the layout in which its
-// reduction stays inside one thread:
-//   pass 1  D[row][key] = Q . K_tile^T, queries as the A operand in TMEM
-//           (staged there by the epilogue warps); a thread owns a row and
-//           folds its keys into the row's running max and sum;
-//   pass 2  D[key][row] = K_tile . Q^T, key tile as the A operand and the
-//           queries as the B operand in shared memory (one 32 KB buffer,
-//           loaded by TMA per item); a thread owns a key and sums its 128
+// One persistent CTA per SM, item i on CTA i mod grid; in its step k a CTA
+// runs P1(a_k) then P2(a_k-1), so that keys are re-read from L2 one item
+// after their first read; a publisher warp merges pass-1 row statistics.
+// Each pass takes the layout in which its reduction stays inside one thread:
+//   pass 1  D[row][key] = Q . K_tile^T; a thread owns a row and folds its
+//           keys into the row's running max and sum;
+//   pass 2  D[key][row] = K_tile . Q^T; a thread owns a key and sums its 128
 //           rows' probabilities, so a key's vote needs no shuffles and no
 //           exchange between warps.
-// TMEM: three 128-column accumulators and two 64-column query slots. Shared
-// memory: a 5-stage key-tile ring and the pass-2 query buffer.
+// Both passes take the queries from shared memory (a 32 KB buffer per pass,
+// loaded by TMA once per item) and the key tile from a 4-stage TMA ring; TMEM
+// holds four 128-column accumulators, so the MMA issuer can run two tiles
+// ahead of each epilogue warpgroup.
 //
 // Warp roles (352 threads): warp 0 = key-tile and query producer, warp 1 =
 // MMA issuer and TMEM owner, warps 2-9 = two epilogue warpgroups taking
-// alternate tiles (they also stage each item's queries into TMEM, half of the
-// columns each), warp 10 = publisher of pass-1 results. Every wait is bounded; on timeout the
-// CTA raises RIPPLE_ETIMEOUT, every role leaves its loop and TMEM is released.
+// alternate tiles, warp 10 = publisher of pass-1 results. Every wait is
+// bounded; on timeout the CTA raises RIPPLE_ETIMEOUT, every role leaves its
+// loop and TMEM is released.
 #include <cuda.h>
 #include <math.h>
 
@@ -39,14 +37,12 @@ constexpr int kTile = 128;                      // keys per tile
 constexpr int kHalfBytes = kTile * 64 * 2;      // one TMA box: 64 dims of 128 keys
 constexpr int kTileBytes = 2 * kHalfBytes;
 constexpr int kThreads = 352;
-constexpr int kNK = 5;                          // key-tile stages
+constexpr int kNK = 4;                          // key-tile stages
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
-constexpr int kNQ = 2;                          // pass-1 query slots in TMEM (64 columns each)
-constexpr int kNA = 3;                          // accumulators in TMEM (128 columns each)
+constexpr int kNA = 4;                          // accumulators in TMEM (128 columns each)
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
-constexpr uint32_t kQCol = kNA * 128;           // TMEM: accumulators, then query slots
-static_assert(kQCol + kNQ * 64 <= 512, "TMEM columns");
+static_assert(kNA * 128 <= 512, "TMEM columns");
 
 struct Tc1Params {
   int units, upl, T, P, W, Hq, Hkv, G;  // units of all layers, units per layer
@@ -128,7 +124,7 @@ __device__ __forceinline__ void seq_at(const Step &s, int j, int &pass, int &idx
 }
 
 struct Misc {
-  uint64_t k_full[kNK], k_empty[kNK], q_full[kNQ], q_empty[kNQ], acc_full[kNA], acc_empty[kNA];
+  uint64_t k_full[kNK], k_empty[kNK], q_full, q_empty, acc_full[kNA], acc_empty[kNA];
   uint64_t qs_full, qs_empty;           // pass-2 queries in shared memory
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
   uint32_t tmem_base;
@@ -139,7 +135,8 @@ struct Misc {
 };
 
 constexpr int kOffQs = kNK * kTileBytes;          // pass-2 queries: two 64-dim halves
-constexpr int kOffMisc = kOffQs + kTileBytes;
+constexpr int kOffQ1 = kOffQs + kTileBytes;       // pass-1 queries
+constexpr int kOffMisc = kOffQ1 + kTileBytes;
 constexpr int kSmemBytes = kOffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
@@ -202,6 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ktiles = smem;
   uint8_t *qsm = smem + kOffQs;
+  uint8_t *q1m = smem + kOffQ1;
   Misc *ms = (Misc *)(smem + kOffMisc);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = items_of_cta(p);
@@ -211,10 +209,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->k_full[i], 1);
       mbar_init(&ms->k_empty[i], 1);
     }
-    for (int i = 0; i < kNQ; ++i) {
-      mbar_init(&ms->q_full[i], 8);  // both warpgroups' four warps
-      mbar_init(&ms->q_empty[i], 1);
-    }
+    mbar_init(&ms->q_full, 1);
+    mbar_init(&ms->q_empty, 1);
     for (int i = 0; i < kNA; ++i) {
       mbar_init(&ms->acc_full[i], 1);
       mbar_init(&ms->acc_empty[i], 4);
@@ -252,6 +248,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           {
             int pass, s;
             seq_at(st, j, pass, s);
+            if (pass == 1 && s == 0) {
+              // item k's queries into the pass-1 buffer, once the previous
+              // item's pass-1 MMAs have read it
+              if (!wait_bar(&ms->q_empty, (k & 1) ^ 1, ms, p.status)) {
+                ok = false;
+                break;
+              }
+              const int layer = st.u1 / p.upl, local = st.u1 % p.upl;
+              const int b = local / p.Hkv, h = local % p.Hkv;
+              const int qrow0 = (b * p.Hq + h * p.G) * p.W;
+              mbar_arrive_expect_tx(&ms->q_full, kTileBytes);
+              tma_load_2d(q1m, &lp.qmap[layer], 0, qrow0, &ms->q_full);
+              tma_load_2d(q1m + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->q_full);
+            }
             if (pass == 2 && s == 0) {
               // the pass-2 item's queries (rows of its unit) into shared memory
               if (!wait_bar(&ms->qs_empty, (qcount & 1) ^ 1, ms, p.status)) {
@@ -293,24 +303,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int kcount = 0, acount = 0, qcount = 0;
       constexpr uint32_t id = idesc_bf16(128, 128);
-      const uint32_t kbase = smem_u32(ktiles), qsbase = smem_u32(qsm);
+      const uint32_t kbase = smem_u32(ktiles), qsbase = smem_u32(qsm), q1base = smem_u32(q1m);
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
-        const int qs1 = k % kNQ;
-        if (k < n && !wait_bar(&ms->q_full[qs1], (k / kNQ) & 1, ms, p.status)) break;
+        if (k < n && !wait_bar(&ms->q_full, k & 1, ms, p.status)) break;
         for (int j = 0; j < st.len && ok; ++j) {
           {
             int pass, s;
             seq_at(st, j, pass, s);
             if (pass == 2 && s == 0) {
-              if (st.n1 > 0) mma_commit(&ms->q_empty[qs1]);  // item k's TMEM queries are free
+              if (st.n1 > 0) mma_commit(&ms->q_empty);  // item k's pass-1 queries are free
               if (!wait_bar(&ms->qs_full, qcount & 1, ms, p.status)) {
                 ok = false;
                 break;
               }
             }
-            const uint32_t qa = tmem + kQCol + qs1 * 64;
             const int ks = kcount % kNK, as = acount % kNA;
             if (!wait_bar(&ms->k_full[ks], (kcount / kNK) & 1, ms, p.status) ||
                 !wait_bar(&ms->acc_empty[as], ((acount / kNA) & 1) ^ 1, ms, p.status)) {
@@ -322,10 +330,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t ka = kbase + ks * kTileBytes;
             if (pass == 1) {
 #pragma unroll
-              for (int kk = 0; kk < 8; ++kk)
-                mma_bf16_tmem_a(d, qa + kk * 8,
-                                sw128_desc(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32), id,
-                                kk > 0);
+              for (int kk = 0; kk < 8; ++kk) {
+                const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+                mma_bf16(d, sw128_desc(q1base + off), sw128_desc(ka + off), id, kk > 0);
+              }
             } else {
 #pragma unroll
               for (int kk = 0; kk < 8; ++kk) {
@@ -343,7 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(&ms->qs_empty);  // the pass-2 queries are free
           ++qcount;
         } else if (ok && st.n1 > 0) {
-          mma_commit(&ms->q_empty[qs1]);  // no pass-2 tiles: item k's TMEM queries are free
+          mma_commit(&ms->q_empty);  // no pass-2 tiles: item k's pass-1 queries are free
         }
       }
       mma_commit(&ms->mma_done);
@@ -411,39 +419,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     int tcount = 0;  // tiles seen
 
-    // Stages item k's window queries into query slot k % kNQ: this thread's
-    // row, this warpgroup's half of the 64 columns.
-    auto load_q = [&](int k) {
-      const int qs = k % kNQ;
-      warp_wait(&ms->q_empty[qs], ((k / kNQ) & 1) ^ 1, ms, p.status);
-      tc_fence_after();
-      const ItemRef it = item_of(p, k);
-      const int layer = it.unit / p.upl, local = it.unit % p.upl;
-      const int b = local / p.Hkv, h = local % p.Hkv;
-      const size_t row = (size_t)(b * p.Hq + h * p.G) * p.W + r;
-      const uint4 *src = reinterpret_cast<const uint4 *>(p.q[layer] + row * 256 + wg * 128);
-      uint32_t w[32];
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 u = __ldg(src + c);
-        w[4 * c] = u.x;
-        w[4 * c + 1] = u.y;
-        w[4 * c + 2] = u.z;
-        w[4 * c + 3] = u.w;
-      }
-      tmem_st32(tmem + lane_addr + kQCol + qs * 64 + wg * 32, w);
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ms->q_full[qs]);
-    };
-
-    if (n > 0) load_q(0);
     // Inside an item every warp follows the same control flow even if a wait
     // gives up (the tile is then skipped), so that the named barriers below
     // are always reached by all of their threads.
     for (int k = 0; k < n + kLag; ++k) {
-      if (k + 1 < n) load_q(k + 1);
       const Step st = step_of(p, k, n);
       float m = -INFINITY, l = 0.f;    // pass 1 of item k: this row's max and sum
       const int last_vis = p.P + r % p.W;
