@@ -59,11 +59,13 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU seconds of the oracle sample")
-    ap.add_argument("--case", choices=["compress", "decode", "perturb", "kl"], default=None,
+    ap.add_argument("--case", choices=["compress", "decode", "perturb", "kl", "serve"],
+                    default=None,
                     help="time one entry point alone (one layer / one decode step / the "
                          "profiling kernels: Eq. 6 perturbation of one layer's V cache, Eq. 7 "
-                         "window KL of every layer's perturbed run), e.g. as a small ncu "
-                         "target; prints one JSON line")
+                         "window KL of every layer's perturbed run; serve: the per-layer "
+                         "decode loop with stand-in projections in a CUDA graph), e.g. as a "
+                         "small ncu target; prints one JSON line")
     ap.add_argument("--vocab", type=int, default=128256,
                     help="--case kl: vocabulary size (128256: Llama-3)")
     ap.add_argument("--repeat", type=int, default=10, help="calls timed in --case mode")
@@ -96,6 +98,11 @@ def run_case(args):
     times = []
     if args.case in ("perturb", "kl"):
         return run_profile_case(args, R, synth, wl, dev)
+    if args.case == "serve":
+        line = {"case": "serve", "workload": wl.name}
+        line.update(serving_loop_measure(R, synth, wl, dev, min(args.repeat * 4, wl.decode_steps)))
+        print(json.dumps(line), flush=True)
+        return
     if args.case == "compress":
         layer = max(range(L), key=lambda i: budgets[i])
         q_win = synth.layer_window_queries(wl, layer, dev)
@@ -226,6 +233,89 @@ def run_profile_case(args, R, synth, wl, dev):
                       "ms_per_call": round(ms, 5), "bytes_per_call": nbytes,
                       "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
                       "peak_source": src}), flush=True)
+
+
+def serving_loop_measure(R, synth, wl, dev, steps):
+    """The per-layer serving shape (Sec. 4.1; Table 3's decode): every layer
+    calls ripple_decode_attn on its own cache between stand-in projections
+    (torch matmuls hidden -> q/k/v and attention output -> hidden; not the
+    method), one step of all layers captured in a CUDA graph and replayed per
+    token. Returns ms per token step of the whole loop, of the same graph
+    without the projections (per-layer decode launches only) and of the
+    all-layers decode launch on the same caches."""
+    import torch
+
+    from paper_2608_08684_gb300.serving import LayerDecodeLoop
+    L, B, Hq, Hkv, d = wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim
+    dt = wl.torch_dtype
+    budgets = R.ripple_alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
+                                     wl.global_budget)
+    n_keep = [R.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets]
+    warm = 3
+    caps = [n + 2 * (steps + warm) + 2 for n in n_keep]
+    kc, vc = zip(*[synth.decode_caches(wl, l, caps[l], dev) for l in range(L)])
+    kc, vc = list(kc), list(vc)
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    hid = Hq * d
+    h = torch.randn(B, hid, generator=g, device=dev).to(dt)
+    wqkv = [(torch.randn(hid, (Hq + 2 * Hkv) * d, generator=g, device=dev) / hid ** 0.5).to(dt)
+            for _ in range(L)]
+    wo = [(torch.randn(hid, hid, generator=g, device=dev) / hid ** 0.5).to(dt) for _ in range(L)]
+    qb = torch.zeros(1, B, Hq, d, dtype=dt, device=dev)
+    kb = torch.zeros(1, B, Hkv, d, dtype=dt, device=dev)
+    vb = torch.zeros(1, B, Hkv, d, dtype=dt, device=dev)
+
+    def before(l):
+        hn = h.float()
+        x = (hn * torch.rsqrt(hn.square().mean(-1, keepdim=True) + 1e-6)).to(dt) @ wqkv[l]
+        qb.copy_(x[:, :Hq * d].reshape(1, B, Hq, d))
+        kb.copy_(x[:, Hq * d:(Hq + Hkv) * d].reshape(1, B, Hkv, d))
+        vb.copy_(x[:, (Hq + Hkv) * d:].reshape(1, B, Hkv, d))
+        return qb, kb, vb
+
+    def after(l, out):
+        h.add_(out.reshape(B, hid).to(dt) @ wo[l])
+
+    def timed(fn, n):
+        for _ in range(warm):
+            fn()
+        torch.cuda.synchronize()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(n):
+            fn()
+        b_.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b_) / n
+
+    lens = torch.tensor(n_keep, dtype=torch.int32, device=dev)
+    full = LayerDecodeLoop(kc, vc, lens, Hq, before, after)
+    full.issue_step()
+    full.capture()
+    ms_full = timed(full.replay, steps)
+    lens.copy_(torch.tensor(n_keep, dtype=torch.int32, device=dev))
+    attn = LayerDecodeLoop(kc, vc, lens, Hq, lambda l: (qb, kb, vb), lambda l, o: None)
+    attn.issue_step()
+    attn.capture()
+    ms_attn = timed(attn.replay, steps)
+    assert int(full.status.item()) == 0 and int(attn.status.item()) == 0
+    # the all-layers launch on the same caches (one decode kernel per step)
+    lens.copy_(torch.tensor(n_keep, dtype=torch.int32, device=dev))
+    ddesc = R.decode_desc(L, B, Hq, Hkv, d, dt)
+    tables = R.DecodeTables(kc, vc)
+    dws = torch.empty(R.ripple_decode_workspace_bytes(ddesc, caps), dtype=torch.uint8, device=dev)
+    q, kn, vn = synth.decode_inputs(wl, 0, dev)
+    out = torch.empty(L, B, Hq, d, device=dev)
+    ms_one = timed(lambda: R.ripple_decode_attn(ddesc, q, kn, vn, tables, lens, out, dws), steps)
+    return {"steps": steps, "ms_per_token_step": round(ms_full, 4),
+            "tokens_per_s": round(B / (ms_full / 1e3), 1),
+            "per_layer_decode_launches_ms_per_step": round(ms_attn, 4),
+            "all_layers_one_launch_ms_per_step": round(ms_one, 4),
+            "what": (f"{L} layers x (stand-in q/k/v projection, single-layer ripple_decode_attn "
+                     f"appending, stand-in output projection) per token, CUDA graph replayed "
+                     f"{steps} times; caches at the RippleKV sizes ({min(n_keep)}..{max(n_keep)} "
+                     f"rows)")}
 
 
 def profile_traffic(profile, sources, alg_bytes):

@@ -2,7 +2,7 @@
 // query attends to the cached states), with the append of the new token.
 //
 // One persistent launch per step covers every layer; one CTA per SM with 8
-// compute warps and one producer warp. Work item = up to kItemRows cache rows
+// compute warps and one producer warp. Work item = up to p.item_rows cache rows
 // of one (layer, batch row, KV head) group; items are fetched with an atomic
 // counter (one ahead), layers with the longest caches first. The producer
 // stages each item's G query rows and then its sub-chunks of K and V rows in
@@ -96,7 +96,7 @@ struct DecCfg {
   static constexpr int STAGES =
       cmin(kMaxStages, (kSmemBudget - kMiscBytes - kItemSlots * QBYTES - (kWarps + 2) * G * D * 4) /
                            (2 * STAGE_BYTES));
-  static_assert(kItemRows % CR == 0, "items are whole sub-chunks");
+  static_assert(kMinItemRows % CR == 0, "items are whole sub-chunks");
   static_assert(S <= 32 && S <= NPIECE && NPIECE % S == 0, "lanes per row");
   static_assert(STAGE_BYTES <= kMaxStageBytes, "stage size");
   static_assert(DL % 2 == 0 && PE % 2 == 0, "fp32x2 pairs");
@@ -144,9 +144,9 @@ __device__ __forceinline__ ItemInfo item_info(const DecParams &p, const S &s, in
   f.group = (f.layer * p.B + f.b) * p.Hkv + f.h;
   f.len = s.len[lo];
   f.full = f.len < 0;
-  f.r0 = f.chunk * kItemRows;
+  f.r0 = f.chunk * p.item_rows;
   // rows 0..len: the cached rows and the new token
-  f.rows = f.full ? 0 : min(kItemRows, f.len + 1 - f.r0);
+  f.rows = f.full ? 0 : min(p.item_rows, f.len + 1 - f.r0);
   return f;
 }
 
@@ -622,14 +622,14 @@ __device__ __forceinline__ void prefetch_first_item(const DecParams &p) {
     const int l = p.order[t];
     const int len = *(volatile const int32_t *)&p.lens[l];
     const bool full = len < 0 || len >= p.cap[l];
-    const int nch = full ? 1 : (len + 1 + kItemRows - 1) / kItemRows;
+    const int nch = full ? 1 : (len + p.item_rows) / p.item_rows;
     if (rest >= units * nch) {
       rest -= units * nch;
       continue;
     }
     if (full) return;
     const int unit = rest / nch, chunk = rest % nch;
-    const int r0 = chunk * kItemRows, r1 = min(len, r0 + kItemRows);
+    const int r0 = chunk * p.item_rows, r1 = min(len, r0 + p.item_rows);
     const int rows = min(r1 - r0, C::STAGES * C::CR);
     if (rows <= 0) return;
     const size_t off = ((size_t)unit * p.cap[l] + r0) * C::ROW_BYTES;
@@ -661,7 +661,7 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     const int len = p.lens[l];
     const bool full = len < 0 || len >= p.cap[l];
     s.len[tid] = full ? -1 : len;
-    s.nch[tid] = full ? 1 : (len + 1 + kItemRows - 1) / kItemRows;
+    s.nch[tid] = full ? 1 : (len + p.item_rows) / p.item_rows;
     if (full && blockIdx.x == 0) report(p.status, RIPPLE_EFULL);
   }
   if (tid == 0) {
@@ -795,7 +795,27 @@ int next_epoch() {
 }
 
 // Cache rows per work item (the workspace holds one partial per item).
-int item_rows(const ripple_decode_desc *) { return kItemRows; }
+// Cache rows per work item for these capacities: kMaxItemRows when that
+// already gives at least one item per SM; otherwise (a single layer's step,
+// short caches) the smallest power of two down to kMinItemRows whose items
+// still fit in one wave of one CTA per SM, so that no CTA takes two items one
+// after the other. A step's lengths are at most its capacities, so the plan's
+// item count bounds the kernel's.
+int item_rows(const ripple_decode_desc *d, const int32_t *caps) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  const long long sms = sm_count(dev);
+  auto items = [&](int rows) {
+    long long n = 0;
+    for (int l = 0; l < d->n_layers; ++l)
+      n += (long long)d->batch * d->n_kv_heads * ((caps[l] + rows - 1) / rows);
+    return n;
+  };
+  int rows = kMaxItemRows;
+  if (items(rows) >= sms) return rows;
+  while (rows > kMinItemRows && items(rows / 2) <= sms) rows /= 2;
+  return rows;
+}
 
 static size_t round_up(size_t x) { return (x + 255) & ~(size_t)255; }
 
@@ -803,7 +823,7 @@ static size_t round_up(size_t x) { return (x + 255) & ~(size_t)255; }
 // partial outputs. Returns the total bytes; fills p's pointers if given.
 size_t plan(const ripple_decode_desc *d, const int32_t *caps, void *ws, DecParams *p) {
   const int G = d->n_q_heads / d->n_kv_heads;
-  const int rows = item_rows(d);
+  const int rows = item_rows(d, caps);
   size_t items = 0;
   for (int l = 0; l < d->n_layers; ++l)
     items += (size_t)d->batch * d->n_kv_heads * ((caps[l] + rows - 1) / rows);
@@ -813,6 +833,7 @@ size_t plan(const ripple_decode_desc *d, const int32_t *caps, void *ws, DecParam
   const size_t o = round_up(sizeof(float) * items * G * d->head_dim);
   if (p != nullptr) {
     uint8_t *base = (uint8_t *)ws;
+    p->item_rows = rows;
     p->ctrl = (int *)base;
     p->ws_ml = (float2 *)(base + ctrl);
     p->ws_o = (float *)(base + ctrl + ml);

@@ -22,13 +22,18 @@ struct DecParams {
   int epoch;        // nonzero tag of this call: the init flag's value once the
                     // counters are zeroed
   long long wait_cycles;  // bound of the in-kernel waits
+  int item_rows;          // cache rows per work item
   const void *kc[RIPPLE_MAX_LAYERS];
   const void *vc[RIPPLE_MAX_LAYERS];
   int cap[RIPPLE_MAX_LAYERS];
   int order[RIPPLE_MAX_LAYERS];  // layers by decreasing capacity
 };
 
-constexpr int kItemRows = 4096;  // cache rows per work item
+// Cache rows per work item: kMaxItemRows, or for steps with fewer such items
+// than SMs (a single layer's step, short caches) smaller items, down to
+// kMinItemRows, as long as they fit in one wave.
+constexpr int kMaxItemRows = 4096;
+constexpr int kMinItemRows = 256;
 
 // Control block of a step in the workspace (int32 words). The init flag has a
 // 128-byte line to itself; CTA 0 zeroes the counters at the start of every

@@ -12,7 +12,8 @@ SCORE_RTOL = 1e-3      # votes: relative, fp32 accumulation from bf16/fp32 input
 SCORE_ATOL_REL = 1e-9  # absolute floor, relative to the largest vote (underflow guard)
 SELECT_GAP_RTOL = 2e-3  # a set mismatch needs two votes within 2x the score tolerance
 DECODE_ATOL = 2e-2     # decode output, max-abs against the fp64 oracle (acceptance bar)
-# Decode output, max-abs: the kernel's own precision. Inputs are exact in fp32;
+# Decode output, max-abs: the kernel's own precision, for values of unit scale
+# (every test draws or normalises them so). Inputs are exact in fp32;
 # each lane sums its share of a group's rows (at most a few hundred terms of
 # |p v| <= |v|, |v| < 6) in fp32 and the shares merge through short trees, with
 # exponentials of relative error ~2^-22: a worst case of a few 1e-5, observed

@@ -66,10 +66,14 @@ DECODE_SHAPES = [
                           dtype="bf16", seed=42), [127, 513]),
     ("bf16-d64-G1", dict(n_layers=2, batch=2, n_q_heads=3, n_kv_heads=3, head_dim=64,
                          dtype="bf16", seed=43), [64, 200]),
-    # groups split over several work items (4096 rows each), item edges and a ragged tail
+    # groups split over several work items, item edges and a ragged tail: with
+    # few groups the items shrink to 256 rows (fewer items than SMs otherwise)
     ("bf16-d128-G4-split", dict(n_layers=4, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
                                 dtype="bf16", kv_dist="scaled_sinks", seed=47),
      [2047, 4096, 4097, 8300]),
+    # with enough groups the items keep 4096 rows
+    ("bf16-d128-G4-split4096", dict(n_layers=2, batch=4, n_q_heads=32, n_kv_heads=8,
+                                    head_dim=128, dtype="bf16", seed=53), [4097, 8300]),
     ("bf16-d128-G1", dict(n_layers=2, batch=2, n_q_heads=2, n_kv_heads=2, head_dim=128,
                           dtype="bf16", seed=48), [0, 129]),
     ("bf16-d128-G2", dict(n_layers=2, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=128,
