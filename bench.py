@@ -57,6 +57,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the other workloads and the serving-loop measurement")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU seconds of the oracle sample")
     ap.add_argument("--case", choices=["compress", "decode", "perturb", "kl", "serve"],
@@ -513,6 +515,79 @@ class Serving:
         return tot / wl.decode_steps
 
 
+def measure_workloads(R, synth, dev, names, reps):
+    """The serving step on other workloads (each generated, timed and freed in
+    turn): compression of all layers and decode steps, with their fractions of
+    the measured HBM bandwidth; for compression also the tensor-pipe fraction
+    of the window-query contraction (two passes, 2 * G*w * T * d flops per
+    unit and pass) against the measured sustained bf16 peak, and for decode the
+    fp32 FMA fraction (q.k and p.v: 2 * d FMAs per cached row and query head)
+    against the peak derived from the SM count, 128 FMA lanes per SM and the
+    maximum SM clock."""
+    import torch
+    hbm, _ = measured_peaks()
+    tensor_peak = measured_peak("bf16_tflops_sustained", 1700.0)
+    props = torch.cuda.get_device_properties(dev)
+    fma_peak = props.multi_processor_count * 128 * 2 * measured_peak("sm_max_mhz", 2070.0) * 1e6 / 1e12
+    res = {}
+    for name in names:
+        wl = synth.WORKLOADS[name]
+        st = Serving(R, synth, wl, dev)
+        for _ in range(2):
+            st.step()
+        torch.cuda.synchronize()
+        timers = ([], [])
+        for _ in range(reps):
+            st.step(timers)
+        torch.cuda.synchronize()
+        assert int(st.status.item()) == 0
+        comp = statistics.mean(elapsed_ms(timers[0]))
+        dec = statistics.mean(elapsed_ms(timers[1])) / wl.decode_steps
+        R_rows, units = wl.group * wl.window, wl.batch * wl.n_kv_heads
+        flops = sum(4.0 * R_rows * wl.seq_len * wl.head_dim * units
+                    for n in st.n_keep if n < wl.seq_len)
+        fmas = sum(units * (n + t + 1) * wl.group * 2 * wl.head_dim
+                   for t in range(wl.decode_steps) for n in st.n_keep) / wl.decode_steps
+        cg = st.compress_bytes() / (comp / 1e3) / 1e9
+        dg = st.decode_bytes_per_step() / (dec / 1e3) / 1e9
+        res[name] = {"workload": wl.name, "dtype": wl.dtype,
+                     "compress_ms": round(comp, 4), "compress_gbs": round(cg, 1),
+                     "compress_frac_hbm": round(cg / hbm, 4),
+                     "compress_tokens_per_s": round(wl.batch * wl.seq_len / (comp / 1e3), 1),
+                     "compress_tensor_tflops": round(flops / (comp / 1e3) / 1e12, 1),
+                     "compress_frac_tensor_sustained": round(flops / (comp / 1e3) / 1e12 / tensor_peak, 4),
+                     "decode_ms_per_step": round(dec, 5), "decode_gbs": round(dg, 1),
+                     "decode_frac_hbm": round(dg / hbm, 4),
+                     "decode_fma_tflops": round(2 * fmas / (dec / 1e3) / 1e12, 2),
+                     "decode_frac_fma_peak": round(2 * fmas / (dec / 1e3) / 1e12 / fma_peak, 4),
+                     "step_ms": round(comp + dec * wl.decode_steps, 3),
+                     "reps": reps}
+        del st
+        torch.cuda.empty_cache()
+    res["peaks"] = {"hbm_gbs": hbm, "bf16_tflops_sustained": tensor_peak,
+                    "fp32_fma_tflops_derived": round(fma_peak, 1)}
+    return res
+
+
+def measured_peak(key, fallback):
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)[key])
+    except Exception:
+        return fallback
+
+
+def workload_config(wl, world, budgets):
+    """The `config` object of a bench line (both arms report the same one)."""
+    return {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch,
+            "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
+            "seq_len": wl.seq_len, "window": wl.window, "pool_kernel": wl.pool_kernel,
+            "ratio": wl.ratio, "avg_budget": wl.avg_budget, "decode_steps": wl.decode_steps,
+            "budgets": list(budgets), "parallelism": f"replicas{world}",
+            "l2": "inputs larger than L2 (K+V per layer %.0f MB), no flush"
+                  % (2 * wl.batch * wl.n_kv_heads * wl.seq_len * wl.head_dim * wl.elem_bytes / 1e6)}
+
+
 def elapsed_ms(pairs):
     return [a.elapsed_time(b) for a, b in pairs]
 
@@ -636,6 +711,18 @@ def run_ours(args, rank, world, local_rank):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(st, args.cpu_seconds)
+    budgets = st.budgets
+    others = serving = None
+    if rank == 0 and world == 1 and not args.no_workloads:
+        # the other workloads and the per-layer serving loop, after the
+        # headline workload's buffers are freed
+        del st, timers
+        torch.cuda.empty_cache()
+        with ClockSampler(gpu_index) as oclocks:
+            others = measure_workloads(R, synth, device,
+                                       [n for n in synth.WORKLOADS if n != args.workload], 3)
+            serving = serving_loop_measure(R, synth, wl, device, 32)
+        others["clocks"] = oclocks.summary()
     if rank != 0:
         return
     line = {
@@ -643,15 +730,7 @@ def run_ours(args, rank, world, local_rank):
         "value": round(value, 1), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch,
-                   "q_heads": wl.n_q_heads, "kv_heads": wl.n_kv_heads, "head_dim": wl.head_dim,
-                   "seq_len": wl.seq_len, "window": wl.window, "pool_kernel": wl.pool_kernel,
-                   "ratio": wl.ratio, "avg_budget": wl.avg_budget,
-                   "decode_steps": wl.decode_steps, "budgets": st.budgets,
-                   "parallelism": f"replicas{world}",
-                   "l2": "inputs larger than L2 (K+V per layer %.0f MB), no flush"
-                         % (2 * wl.batch * wl.n_kv_heads * wl.seq_len * wl.head_dim
-                            * wl.elem_bytes / 1e6)},
+        "config": workload_config(wl, world, budgets),
         "compress": {"tokens_per_s": round(tokens / world / (comp_avg / 1e3), 1),
                      "ms": round(comp_avg, 4), "gbs": round(comp_gbs, 1),
                      "frac_hbm": round(comp_gbs / hbm, 4),
@@ -667,6 +746,9 @@ def run_ours(args, rank, world, local_rank):
     }
     if e2e:
         line["e2e"] = e2e
+    if others:
+        line["workloads"] = others
+        line["serving_loop"] = serving
     if cpu:
         line["cpu_baseline"] = cpu
     print(json.dumps(line), flush=True)
@@ -721,140 +803,148 @@ def measure_e2e(st, args, torch, tokens):
 # ----------------------------------------------------------------- CPU oracle
 
 
-def oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, target_s, layers=None):
-    """Times the oracle on a bounded sample of compression units and decode
-    groups and extrapolates to one full step. Returns (step seconds, sample text).
-    `layers` limits the compression sample to those layers (all by default)."""
-    import numpy as np
-
-    from oracle import ripple_oracle as O
-    scale = 1.0 / math.sqrt(wl.head_dim)
-    units_total = wl.n_layers * wl.batch * wl.n_kv_heads
-    # compression sample: units round robin over the sampled layers (each
-    # layer's own budget), then over (b, h), until about 3/4 of the time target
-    layers = list(range(wl.n_layers)) if layers is None else list(layers)
-    t_comp, n_comp = 0.0, 0
-    while t_comp < 0.75 * target_s and n_comp < len(layers) * wl.batch * wl.n_kv_heads:
-        layer = layers[n_comp % len(layers)]
-        b, h = divmod((n_comp // len(layers)) % (wl.batch * wl.n_kv_heads), wl.n_kv_heads)
-        q, k, v = get_unit(layer, b, h)
-        t = time.perf_counter()
-        O.compress_unit(q, k, v, budgets[layer], wl.window, scale, wl.pool_kernel)
-        t_comp += time.perf_counter() - t
-        n_comp += 1
-    # decode sample: one (layer, b, h) group per layer, over the first steps
-    steps = min(16, wl.decode_steps)
-    t_dec, n_dec = 0.0, 0
-    for layer in range(wl.n_layers):
-        if t_dec > 0.25 * target_s:
-            break
-        kk, vv, qs, kns, vns = get_decode(layer, steps)
-        rows_k, rows_v = kk, vv
-        t = time.perf_counter()
-        for s in range(steps):
-            rows_k = np.vstack([rows_k, kns[s][None]])
-            rows_v = np.vstack([rows_v, vns[s][None]])
-            O.decode_attention(qs[s], rows_k, rows_v, scale)
-        t_dec += time.perf_counter() - t
-        n_dec += steps
-    per_unit = t_comp / n_comp
-    per_group_step = t_dec / n_dec
-    step_s = per_unit * units_total + per_group_step * (
-        wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps)
-    sample = (f"{n_comp} compression units (T={wl.seq_len}, round robin over {len(layers)} "
-              f"layers) and {n_dec} "
-              f"decode (group, step) pairs; extrapolated to {units_total} units and "
-              f"{wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps} group-steps")
-    return step_s, sample, t_comp + t_dec
+# ----------------------------------------------------------------- CPU oracle
+#
+# The oracle is timed on a bounded sample of the workload by a pool of worker
+# processes (spawned, one BLAS/torch thread each, one per host core); each
+# worker regenerates its layer's seeded inputs on the host, then times whole
+# compression units (compress_unit) and decode steps of single groups
+# (decode_attention) until its time budget is spent. The full step's time is
+# extrapolated from the pool's aggregate rates: a reported baseline only.
 
 
-def _decode_sampler(wl, n_keep):
-    """Seeded decode inputs of one (layer, b=0, h=0) group on the host: a cache
-    of the layer's retained length and the first decode steps' rows."""
-    from paper_2608_08684_gb300 import synth
-    G = wl.group
-
-    def get(layer, steps):
-        one = wl.replace(batch=1, n_kv_heads=1, n_q_heads=G)
-        kc, vc = synth.decode_caches(one, layer, n_keep[layer])
-        dec = [synth.decode_inputs(one, s, layers=[layer]) for s in range(steps)]
-        return (synth.to_f64(kc[0, 0]), synth.to_f64(vc[0, 0]),
-                [synth.to_f64(d[0][0, 0]) for d in dec], [synth.to_f64(d[1][0, 0, 0]) for d in dec],
-                [synth.to_f64(d[2][0, 0, 0]) for d in dec])
-    return get
+def _oracle_worker_init():
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[var] = "1"
 
 
-def _threads():
-    try:
-        import threadpoolctl
-        info = threadpoolctl.threadpool_info()
-        n = max((i.get("num_threads", 1) for i in info), default=1)
-        return int(n)
-    except Exception:
-        return os.cpu_count() or 1
-
-
-def cpu_baseline(st, target_s):
-    import numpy as np
-
-    from paper_2608_08684_gb300 import synth
-    wl = st.wl
-    G = wl.group
-
-    def get_unit(layer, b, h):
-        return (synth.to_f64(st.q_win[layer][b, h * G:(h + 1) * G]), synth.to_f64(st.k[layer][b, h]),
-                synth.to_f64(st.v[layer][b, h]))
-
-    get_decode = _decode_sampler(wl, st.n_keep)
-
-    step_s, sample, spent = oracle_sample_time(wl, get_unit, get_decode, st.budgets, st.n_keep,
-                                               target_s)
-    return {"value": round(wl.batch * wl.seq_len / step_s, 2), "unit": "tokens/s",
-            "cores": _threads(), "kind": "oracle", "sample": sample,
-            "sample_seconds": round(spent, 2), "step_seconds_extrapolated": round(step_s, 2)}
-
-
-def run_reference(args, rank, world):
-    """Reference arm: the CPU oracle, timed on this host's cores, each step a
-    bounded sample of the workload extrapolated to a full step."""
-    if rank != 0:
-        return
+def _oracle_worker(task):
+    """One sampling task in a worker process: ("compress", workload fields,
+    layer, budget, [(b, h), ...], seconds) or ("decode", workload fields,
+    layer, n_keep, steps, seconds). Returns (units or group-steps done, compute
+    seconds)."""
     import numpy as np
     import torch
 
     from oracle import ripple_oracle as O
     from paper_2608_08684_gb300 import synth
+    torch.set_num_threads(1)
+    kind, fields, layer = task[0], task[1], task[2]
+    wl = synth.Workload(**fields)
+    G, scale = wl.group, 1.0 / math.sqrt(wl.head_dim)
+    if kind == "compress":
+        budget, units, seconds = task[3], task[4], task[5]
+        q = synth.layer_window_queries(wl, layer)
+        k = synth.layer_keys(wl, layer)
+        v = synth.layer_values(wl, layer)
+        done, spent = 0, 0.0
+        for b, h in units:
+            if spent >= seconds:
+                break
+            qu = synth.to_f64(q[b, h * G:(h + 1) * G])
+            ku, vu = synth.to_f64(k[b, h]), synth.to_f64(v[b, h])
+            t = time.perf_counter()
+            O.compress_unit(qu, ku, vu, budget, wl.window, scale, wl.pool_kernel)
+            spent += time.perf_counter() - t
+            done += 1
+        return done, spent
+    n_keep, steps, seconds = task[3], task[4], task[5]
+    one = wl.replace(batch=1, n_kv_heads=1, n_q_heads=G)
+    kc, vc = synth.decode_caches(one, layer, n_keep)
+    rows_k, rows_v = synth.to_f64(kc[0, 0]), synth.to_f64(vc[0, 0])
+    done, spent = 0, 0.0
+    for s in range(steps):
+        if spent >= seconds:
+            break
+        q, kn, vn = synth.decode_inputs(one, s, layers=[layer])
+        qq, kk, vv = synth.to_f64(q[0, 0]), synth.to_f64(kn[0, 0, 0]), synth.to_f64(vn[0, 0, 0])
+        t = time.perf_counter()
+        rows_k = np.vstack([rows_k, kk[None]])
+        rows_v = np.vstack([rows_v, vv[None]])
+        O.decode_attention(qq, rows_k, rows_v, scale)
+        spent += time.perf_counter() - t
+        done += 1
+    return done, spent
+
+
+def oracle_step_time(wl, budgets, n_keep, target_s, layers=None, workers=None):
+    """Times the oracle on a bounded sample with a pool of worker processes
+    and extrapolates to one full step. Returns a dict with the step seconds,
+    the worker count, the sampled fraction and a description."""
+    import multiprocessing as mp
+    workers = workers or os.cpu_count() or 1
+    layers = list(range(wl.n_layers)) if layers is None else list(layers)
+    fields = dict(wl.__dict__)
+    units_all = [(b, h) for b in range(wl.batch) for h in range(wl.n_kv_heads)]
+    # compression: one task per worker, round robin over the sampled layers,
+    # each task taking a strided share of its layer's units
+    per_layer = max(1, workers // len(layers))
+    ctasks = []
+    for i in range(max(workers, len(layers))):
+        layer = layers[i % len(layers)]
+        share = units_all[(i // len(layers)) % per_layer::per_layer]
+        ctasks.append(("compress", fields, layer, budgets[layer], share, 0.75 * target_s))
+    steps = min(16, wl.decode_steps)
+    dtasks = [("decode", fields, layer, n_keep[layer], steps, 0.25 * target_s)
+              for layer in layers[:workers]]
+    t0 = time.perf_counter()
+    with mp.get_context("spawn").Pool(workers, initializer=_oracle_worker_init) as pool:
+        cres = pool.map(_oracle_worker, ctasks, chunksize=1)
+        dres = pool.map(_oracle_worker, dtasks, chunksize=1)
+    wall = time.perf_counter() - t0
+    # aggregate rates: every worker runs in parallel with the others
+    c_rate = sum(d / s for d, s in cres if s > 0)
+    d_rate = sum(d / s for d, s in dres if s > 0)
+    units_total = wl.n_layers * wl.batch * wl.n_kv_heads
+    group_steps = wl.n_layers * wl.batch * wl.n_kv_heads * wl.decode_steps
+    step_s = units_total / c_rate + group_steps / d_rate
+    n_units = sum(d for d, _ in cres)
+    n_dec = sum(d for d, _ in dres)
+    return {"step_s": step_s, "workers": workers, "wall_s": wall,
+            "sample_fraction": (n_units + n_dec) / (units_total + group_steps),
+            "sample": (f"{n_units} compression units (T={wl.seq_len}, {len(layers)} layers "
+                       f"{layers if len(layers) <= 8 else '(evenly spaced)'}) "
+                       f"and {n_dec} decode group-steps timed by {workers} worker processes "
+                       f"(one thread each); extrapolated to {units_total} units and "
+                       f"{group_steps} group-steps by the pool's aggregate rates")}
+
+
+def cpu_baseline(st, target_s):
+    wl = st.wl
+    # one task per worker: evenly spaced layers, at most one per worker
+    workers = os.cpu_count() or 1
+    n = min(workers, wl.n_layers)
+    layers = sorted({round(i * (wl.n_layers - 1) / max(1, n - 1)) for i in range(n)})
+    r = oracle_step_time(wl, st.budgets, st.n_keep, target_s, layers=layers, workers=workers)
+    return {"value": round(wl.batch * wl.seq_len / r["step_s"], 2), "unit": "tokens/s",
+            "cores": r["workers"], "kind": "oracle", "sample": r["sample"],
+            "extrapolated": True, "sample_fraction": round(r["sample_fraction"], 5),
+            "wall_s": round(r["wall_s"], 1),
+            "step_seconds_extrapolated": round(r["step_s"], 2)}
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the CPU oracle, timed on this host's cores (a pool of
+    worker processes), each step a bounded sample of the workload extrapolated
+    to a full step."""
+    if rank != 0:
+        return
+    from oracle import ripple_oracle as O
+    from paper_2608_08684_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
-    G = wl.group
     budgets = O.alloc_budgets(synth.sensitivity_profile(wl), wl.ratio, wl.gamma,
                               wl.global_budget)
     n_keep = [O.keep_count(b, wl.seq_len, wl.window) for b in budgets]
-    # Four sampled layers (largest and smallest budget, two in between), each
-    # generated once on the host.
+    # four sampled layers: largest and smallest budget, two in between
     by_budget = sorted(range(wl.n_layers), key=lambda i: budgets[i])
     sample_layers = sorted({by_budget[-1], by_budget[0], by_budget[len(by_budget) // 3],
                             by_budget[2 * len(by_budget) // 3]})
-    layer_cache = {}
-
-    def layer_tensors(layer):
-        if layer not in layer_cache:
-            layer_cache[layer] = (synth.layer_window_queries(wl, layer),
-                                  synth.layer_keys(wl, layer), synth.layer_values(wl, layer))
-        return layer_cache[layer]
-
-    def get_unit(layer, b, h):
-        q, k, v = layer_tensors(layer)
-        return (synth.to_f64(q[b, h * G:(h + 1) * G]), synth.to_f64(k[b, h]), synth.to_f64(v[b, h]))
-
-    get_decode = _decode_sampler(wl, n_keep)
-
     per_step = max(2.0, min(args.cpu_seconds, 120.0 / max(1, args.steps + args.warmup)))
-    times, sample = [], ""
+    times, r = [], None
     for i in range(args.warmup + args.steps):
-        step_s, sample, _ = oracle_sample_time(wl, get_unit, get_decode, budgets, n_keep, per_step,
-                                               layers=sample_layers)
+        r = oracle_step_time(wl, budgets, n_keep, per_step, layers=sample_layers)
         if i >= args.warmup:
-            times.append(step_s)
+            times.append(r["step_s"])
     step_s = statistics.mean(times)
     value = wl.batch * wl.seq_len / step_s
     line = {"metric": "compressed-prefill tokens/s; ragged decode-attn HBM GB/s vs GB300 peak",
@@ -862,11 +952,15 @@ def run_reference(args, rank, world):
             "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 1),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name},
-            "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": _threads(),
-                             "kind": "oracle", "sample": sample},
+            "config": workload_config(wl, world, budgets),
+            "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": r["workers"],
+                             "kind": "oracle", "sample": r["sample"], "extrapolated": True,
+                             "sample_fraction": round(r["sample_fraction"], 5)},
             "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
-                    "d2h_bytes_per_step": 0}}
+                    "d2h_bytes_per_step": 0},
+            "note": ("each step times a bounded sample of the workload and reports the "
+                     "extrapolated time of a full step; ms_per_step is that extrapolation, "
+                     "not the wall time of the sample")}
     print(json.dumps(line), flush=True)
 
 
