@@ -393,13 +393,22 @@ ripple_status ripple_window_kl_workspace_bytes(int32_t n_sets, int32_t n_pos, in
  * kl_out     fp32 [n_sets][n_pos] per-position divergences, or NULL
  * d_out      fp32 [n_sets] window averages
  * workspace  device scratch of at least ripple_window_kl_workspace_bytes
- *            bytes, 256-byte aligned, no initialisation needed
+ *            bytes, 256-byte aligned; its contents need no initialisation
+ *            (the call zeroes the counters it keeps there); calls that share
+ *            a workspace must be ordered (one stream)
+ * Arithmetic: with delta = q - p, KL = log E_P[exp(delta)] - E_P[delta].
  * Each row is cut into fixed slices of 8192 logits and each slice into fixed
- * shares of 1024; a share is reduced in fp32 to (max, sum of exponentials,
- * P-weighted logit difference) for p and (max, sum) for q, the shares of a
- * row are merged in a fixed order in fp32 and the window mean is summed in
- * double, so results do not depend on the GPU or on the run. Identical p and
- * q rows give exactly 0. The call may be captured in a CUDA graph.
+ * shares of 1024; a share is reduced in fp32 to the sums, over its logits, of
+ * w = exp(p - max p), w x and w (exp(x) - 1 - x) with x = delta - c (c = delta
+ * at the share's first largest p; the last sum by its Taylor polynomial where
+ * |x| <= 1/2 across the share), or of exp(q - r) for a reference r where some
+ * |x| is larger. The shares of a row are merged in double in a fixed order,
+ * KL = log1p(E_P[x] + E_P[exp(x) - 1 - x]) - E_P[x] (so a small divergence
+ * is not the difference of two large terms), and the window mean is summed
+ * in double: results do not depend on the GPU or on the run. Identical p and
+ * q rows give exactly 0. Two kernel launches. The call may be captured in a
+ * CUDA graph; after RIPPLE_ETIMEOUT the outputs are unspecified and a graph
+ * holding the call should be re-captured.
  * Errors: RIPPLE_EINVAL (n_sets < 1, n_pos < 1, bad vocab or dtype, NULL or
  * misaligned pointers), RIPPLE_EWORKSPACE, RIPPLE_ECUDA. Device status:
  * RIPPLE_ETIMEOUT (a bounded in-kernel wait ran out).

@@ -10,12 +10,17 @@ Tolerances, from the fp32 arithmetic of the kernels:
   once to bf16, so it equals the fp64 result rounded to bf16 except where the
   fp64 value lies within that fp32 bound of a rounding midpoint, where the
   two are adjacent bf16 values.
-* window KL: slice statistics in fp32 (exponentials on the special-function
-  unit, relative error about 2^-22 each; sums of at most 8192 terms through
-  32-term thread sums and shuffle trees), combined in double. The sums carry
-  relative errors of about 1e-6, which reach the divergence as absolute
-  errors of a few 1e-6 through log(zq / zp) and the weighted mean of p - q:
-  |gpu - oracle| <= 1e-3 |oracle| + 2e-5.
+* window KL: shares of 1024 logits reduced in fp32 (weights from the
+  special-function exponential, relative error about 2^-22 each; 32-term
+  thread sums and shuffle trees), rows merged in double. Where every share
+  stays in the Taylor regime (|x| <= 1/2) the divergence is formed as
+  log1p(E[x] + E[g(x)]) - E[x]: the weights and the positive sum of g carry
+  relative errors of about 1e-6, and the error of E[x] enters only times
+  E[x] itself, so the error is relative to the divergence:
+  |gpu - oracle| <= 1e-4 |oracle| + 1e-10 at divergences of 1e-5 to 1e-4.
+  Elsewhere the shares' masses are summed in the log domain with relative
+  errors of about 1e-6, which reach the divergence as absolute errors of a
+  few 1e-7 to 1e-6: |gpu - oracle| <= 1e-3 |oracle| + 2e-5.
 """
 import math
 
@@ -30,6 +35,7 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda"
 PERTURB_F32_REL = 2.0 ** -20
 KL_RTOL, KL_ATOL = 1e-3, 2e-5
+KL_SMALL_RTOL, KL_SMALL_ATOL = 1e-4, 1e-10
 
 
 def _perturb_case(lib, B, H, T, d, dtype, pb, pe, in_place, alpha, seed):
@@ -193,6 +199,79 @@ def test_window_kl_large_perturbation_and_without_per_position_output(lib):
         _, d = O.window_kl(synth.to_f64(p), synth.to_f64(q[s]))
         _kl_check([d_out[s].item()], [d])
     assert d_out[0].item() > 1.0 > 1e-3 > d_out[1].item() > 0
+
+
+def test_window_kl_small_divergence_keeps_relative_precision(lib):
+    # perturbations of sigma 0.014 and 0.004: divergences near 1e-4 and 1e-5,
+    # every share in the Taylor regime
+    n_pos, vocab = 8, 128256
+    for dtype in (torch.float32, torch.bfloat16):
+        p, q = synth.window_logits(31, 2, n_pos, vocab, dtype, DEV, sigmas=[0.014, 0.004])
+        ws = torch.empty(lib.ripple_window_kl_workspace_bytes(2, n_pos, vocab),
+                         dtype=torch.uint8, device=DEV)
+        d_out = torch.empty(2, device=DEV)
+        kl_out = torch.empty(2, n_pos, device=DEV)
+        lib.ripple_window_kl(p, q, ws, d_out, kl_out)
+        torch.cuda.synchronize()
+        pp = synth.to_f64(p)
+        for s in range(2):
+            kl, d = O.window_kl(pp, synth.to_f64(q[s]))
+            if dtype == torch.float32:
+                assert 1e-6 < kl.min() and kl.max() < 3e-4
+            got = np.concatenate([kl_out[s].cpu().numpy().astype(np.float64), [d_out[s].item()]])
+            want = np.concatenate([kl, [d]])
+            err = np.abs(got - want)
+            assert np.all(err <= KL_SMALL_RTOL * np.abs(want) + KL_SMALL_ATOL), \
+                (dtype, s, (err / np.abs(want)).max())
+
+
+def test_window_kl_far_logits_and_shifts(lib):
+    n_pos, vocab = 5, 40000
+    p, q = synth.window_logits(32, 4, n_pos, vocab, torch.float32, DEV,
+                               sigmas=[0.01, 0.01, 0.01, 0.01])
+    q[0, :, 17] += 6.0      # two far logits: their shares leave the Taylor regime
+    q[0, :, 30001] -= 9.0
+    q[1, :, 123] += 120.0   # exp(q - q at the largest p) overflows fp32 in that share
+    q[2] = p - 100.0        # constant shift: the same distribution
+    q[3, :, 8191] += 0.75   # one far logit at a slice's last entry
+    ws = torch.empty(lib.ripple_window_kl_workspace_bytes(4, n_pos, vocab), dtype=torch.uint8,
+                     device=DEV)
+    d_out = torch.empty(4, device=DEV)
+    kl_out = torch.empty(4, n_pos, device=DEV)
+    lib.ripple_window_kl(p, q, ws, d_out, kl_out)
+    torch.cuda.synchronize()
+    pp = synth.to_f64(p)
+    for s in range(4):
+        kl, d = O.window_kl(pp, synth.to_f64(q[s]))
+        _kl_check(kl_out[s].cpu().numpy(), kl)
+        _kl_check([d_out[s].item()], [d])
+    assert d_out[1].item() > 50.0 and abs(d_out[2].item()) <= KL_ATOL
+
+
+def test_window_kl_workspace_contents_and_graph_replay(lib):
+    n_sets, n_pos, vocab = 3, 7, 20000
+    p, q = synth.window_logits(33, n_sets, n_pos, vocab, torch.float32, DEV)
+    nbytes = lib.ripple_window_kl_workspace_bytes(n_sets, n_pos, vocab)
+    ref_kl = torch.empty(n_sets, n_pos, device=DEV)
+    ref_d = torch.empty(n_sets, device=DEV)
+    lib.ripple_window_kl(p, q, torch.zeros(nbytes, dtype=torch.uint8, device=DEV), ref_d, ref_kl)
+    # arbitrary workspace contents (every counter word 0xA5A5A5A5)
+    ws = torch.full((nbytes,), 0xA5, dtype=torch.uint8, device=DEV)
+    kl_out = torch.full((n_sets, n_pos), float("nan"), device=DEV)
+    d_out = torch.full((n_sets,), float("nan"), device=DEV)
+    lib.ripple_window_kl(p, q, ws, d_out, kl_out)
+    torch.cuda.synchronize()
+    assert torch.equal(kl_out, ref_kl) and torch.equal(d_out, ref_d)
+    # one call captured in a CUDA graph, replayed twice
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        lib.ripple_window_kl(p, q, ws, d_out, kl_out)
+    for _ in range(2):
+        kl_out.fill_(float("nan"))
+        d_out.fill_(float("nan"))
+        graph.replay()
+        torch.cuda.synchronize()
+        assert torch.equal(kl_out, ref_kl) and torch.equal(d_out, ref_d)
 
 
 def test_window_kl_is_reproducible(lib):
