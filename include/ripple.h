@@ -398,7 +398,7 @@ ripple_status ripple_window_kl_workspace_bytes(int32_t n_sets, int32_t n_pos, in
  *            a workspace must be ordered (one stream)
  * Arithmetic: with delta = q - p, KL = log E_P[exp(delta)] - E_P[delta].
  * Each row is cut into fixed slices of 8192 logits and each slice into fixed
- * shares of 1024; a share is reduced in fp32 to the sums, over its logits, of
+ * shares of 512; a share is reduced in fp32 to the sums, over its logits, of
  * w = exp(p - max p), w x and w (exp(x) - 1 - x) with x = delta - c (c = delta
  * at the share's first largest p; the last sum by its Taylor polynomial where
  * |x| <= 1/2 across the share), or of exp(q - r) for a reference r where some

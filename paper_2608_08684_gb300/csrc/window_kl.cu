@@ -13,7 +13,7 @@
 // so a small divergence keeps its relative precision.
 //
 // Work: every row is cut into slices of kKlSlice logits and every slice into
-// kKlConsumerWarps shares, one per consumer warp (32 logits a lane). A share
+// kKlConsumerWarps shares, one per consumer warp (16 logits a lane). A share
 // is reduced in fp32 to a KlPart: the largest p (mp), the sum of the weights
 // w = exp(p - mp), c = delta at the first largest p, and the sums of w x and
 // of w g(x) -- g by its Taylor polynomial when |x| <= kKlPolyBound across the
@@ -42,7 +42,7 @@
 namespace ripple {
 namespace {
 
-constexpr int kKlConsumerWarps = 8;
+constexpr int kKlConsumerWarps = 16;
 constexpr int kKlThreads = (kKlConsumerWarps + 1) * 32;  // + one producer warp
 constexpr int kKlShareThreads = kKlConsumerWarps * 32;
 constexpr int kKlSlice = 8192;               // logits per work item
@@ -58,7 +58,7 @@ template <typename Tl>
 struct KlCfg {
   static constexpr int V16 = 16 / (int)sizeof(Tl);
   static constexpr int CH = kKlSlice / (kKlShareThreads * V16);
-  static constexpr int E = CH * V16;  // 32 logits
+  static constexpr int E = CH * V16;  // 16 logits
 };
 
 // One consumer warp's share of a slice of a row (see the file comment).
@@ -359,9 +359,9 @@ __device__ __forceinline__ KlRaw load_part(const KlPart *rp, int k, int n) {
   return r;
 }
 
-// Rows of up to kKlMergeCached * 32 partials (vocabularies up to 128
-// slices) are read once into registers; longer rows are read per pass.
-constexpr int kKlMergeCached = 4;
+// Rows of up to kKlMergeCached * 32 partials (vocabularies up to 16 slices,
+// 131072 logits) are read once into registers; longer rows are read per pass.
+constexpr int kKlMergeCached = 8;
 
 template <bool kCached>
 __device__ __forceinline__ double merge_row(const KlPart *rp, int n, int lane) {

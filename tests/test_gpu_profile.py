@@ -10,7 +10,7 @@ Tolerances, from the fp32 arithmetic of the kernels:
   once to bf16, so it equals the fp64 result rounded to bf16 except where the
   fp64 value lies within that fp32 bound of a rounding midpoint, where the
   two are adjacent bf16 values.
-* window KL: shares of 1024 logits reduced in fp32 (weights from the
+* window KL: shares of 512 logits reduced in fp32 (weights from the
   special-function exponential, relative error about 2^-22 each; 32-term
   thread sums and shuffle trees), rows merged in double. Where every share
   stays in the Taylor regime (|x| <= 1/2) the divergence is formed as
