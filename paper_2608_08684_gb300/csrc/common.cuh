@@ -74,6 +74,27 @@ __device__ __forceinline__ void report(int32_t *status, int32_t code) {
   if (status != nullptr) atomicCAS(status, 0, code);
 }
 
+// ------------------------------------------------------- bounds-checked build
+// Compiled with RIPPLE_CHECKED (libripple_checked.so), every guarded global
+// access first tests its offset against the extent of its buffer (both in
+// elements, rows or bytes, as the call site states): an access [off, off +
+// len) outside [0, extent) is reported as RIPPLE_EBOUNDS in the call's status
+// word and moved to offset 0, so it stays inside the buffer and a copy keeps
+// its byte count (no barrier loses bytes); nothing traps. In the normal build
+// guard() is the offset itself.
+#ifdef RIPPLE_CHECKED
+constexpr bool kChecked = true;
+#else
+constexpr bool kChecked = false;
+#endif
+__device__ __forceinline__ long long guard(long long off, long long len, long long extent,
+                                           int32_t *status) {
+  if (!kChecked) return off;
+  if (off >= 0 && len >= 0 && off + len <= extent) return off;
+  report(status, RIPPLE_EBOUNDS);
+  return 0;
+}
+
 // ---------------------------------------------------------------- PTX wrappers
 
 // GPU-scope acquire load / release store of a flag in global memory.

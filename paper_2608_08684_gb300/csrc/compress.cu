@@ -121,13 +121,13 @@ extern "C" ripple_status ripple_compress_layer(const ripple_layer_desc *desc, in
   if (g.P > 0 && (!keep_all || scores_out)) {
     cudaError_t e = score_tc1_supported(g)  ? launch_score_tc1(g, 1, &q_win, &k, ws, votes, dev_status, st)
                     : score_tc_supported(g) ? launch_score_tc(g, q_win, k, ws, votes, dev_status, st)
-                                            : launch_score_simt(g, q_win, k, ws, votes, st);
+                                            : launch_score_simt(g, q_win, k, ws, votes, dev_status, st);
     RIPPLE_CUDA_TRY(e);
   }
   if (keep_all) {
     RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
   } else {
-    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, st));
+    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, dev_status, st));
   }
   RIPPLE_CUDA_TRY(launch_gather(g, 1, &k, &v, &idx_out, &n, &k_out, &v_out, &cap, dev_status, st));
   *n_keep_host = n;
@@ -157,7 +157,7 @@ extern "C" ripple_status ripple_select_layer(const ripple_layer_desc *desc, int6
   if (n == g.T) {
     RIPPLE_CUDA_TRY(launch_iota(g, idx_out, st));
   } else {
-    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, st));
+    RIPPLE_CUDA_TRY(launch_select(g, 1, votes, ws, &n, &idx_out, dev_status, st));
   }
   RIPPLE_CUDA_TRY(launch_gather(g, 1, &k, &v, &idx_out, &n, &k_out, &v_out, &cap, dev_status, st));
   *n_keep_host = n;
@@ -215,7 +215,7 @@ extern "C" ripple_status ripple_compress_layers(
     // All layers in three launches: scoring, selection, gather.
     RIPPLE_CUDA_TRY(launch_score_tc1(g, n_layers, q_win_host, k_host, ws, ws.votes, dev_status,
                                      st));
-    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, st));
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st));
     RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
                                   (const int32_t *const *)idx_out_host, n, k_out_host,
                                   v_out_host, cap, dev_status, st));
@@ -229,10 +229,11 @@ extern "C" ripple_status ripple_compress_layers(
       float *votes_l = ws.votes + (size_t)l * g.units * g.P;
       cudaError_t e = score_tc_supported(g)
                           ? launch_score_tc(g, q_win_host[l], k_host[l], ws, votes_l, dev_status, st)
-                          : launch_score_simt(g, q_win_host[l], k_host[l], ws, votes_l, st);
+                          : launch_score_simt(g, q_win_host[l], k_host[l], ws, votes_l,
+                                              dev_status, st);
       RIPPLE_CUDA_TRY(e);
     }
-    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, st));
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st));
     RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
                                   (const int32_t *const *)idx_out_host, n, k_out_host,
                                   v_out_host, cap, dev_status, st));

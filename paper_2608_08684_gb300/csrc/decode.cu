@@ -311,11 +311,14 @@ __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &
     } else {
       const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
       mbar_arrive_expect_tx(&s.item_full[slot], C::QBYTES);
-      bulk_g2s(s.qs[slot], (const uint8_t *)p.q + qrow * C::ROW_BYTES, C::QBYTES,
+      const long long qr = guard((long long)qrow, G, (long long)p.L * p.B * p.Hq, p.status);
+      bulk_g2s(s.qs[slot], (const uint8_t *)p.q + qr * C::ROW_BYTES, C::QBYTES,
                &s.item_full[slot]);
       const int nsub = (f.rows + C::CR - 1) / C::CR;
       const size_t gbase = (size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer];
-      const size_t nb = ((size_t)f.layer * units + f.b * p.Hkv + f.h) * C::ROW_BYTES;
+      const size_t nb = guard((long long)f.layer * units + f.b * p.Hkv + f.h, 1,
+                              (long long)p.L * units, p.status) *
+                        C::ROW_BYTES;
       for (int sub = 0; sub < nsub; ++sub, ++j) {
         const int stage = j % C::STAGES;
         if (sub == 1 && nxt < 0) nxt = next_of(it);
@@ -329,7 +332,9 @@ __device__ __forceinline__ void produce(const DecParams &p, DecSmem<Tin, D, G> &
         const bool has_new = f.len >= rs && f.len < rs + C::CR;
         mbar_arrive_expect_tx(&s.full[stage], 2u * (nk + (has_new ? 1 : 0)) * C::ROW_BYTES);
         if (nk > 0) {
-          const size_t off = (gbase + rs) * C::ROW_BYTES;
+          const size_t off =
+              guard((long long)(gbase + rs), nk, (long long)units * p.cap[f.layer], p.status) *
+              C::ROW_BYTES;
           bulk_g2s(s.kv[stage][0], (const uint8_t *)p.kc[f.layer] + off, nk * C::ROW_BYTES,
                    &s.full[stage]);
           bulk_g2s(s.kv[stage][1], (const uint8_t *)p.vc[f.layer] + off, nk * C::ROW_BYTES,
@@ -391,7 +396,8 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
     const size_t qrow = ((size_t)f.layer * p.B + f.b) * p.Hq + (size_t)f.h * G;
     if (f.full) {
       if (lane == 0) mbar_arrive(&s.item_empty[slot]);
-      for (int e = tid; e < G * D; e += kWarps * 32) p.out[qrow * D + e] = 0.f;
+      for (int e = tid; e < G * D; e += kWarps * 32)
+        p.out[guard(qrow * D + e, 1, (long long)p.L * p.B * p.Hq * D, p.status)] = 0.f;
       continue;
     }
     __syncwarp();
@@ -502,7 +508,10 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
       // The new token's rows, staged behind the cached rows, go to the cache.
       const int rs = f.r0 + sub * C::CR;
       if (warp == 0 && f.len >= rs && f.len < rs + C::CR) {
-        const size_t dst = ((size_t)(f.b * p.Hkv + f.h) * p.cap[f.layer] + f.len) * C::ROW_BYTES;
+        const size_t dst =
+            guard((long long)(f.b * p.Hkv + f.h) * p.cap[f.layer] + f.len, 1,
+                  (long long)p.B * p.Hkv * p.cap[f.layer], p.status) *
+            C::ROW_BYTES;
         for (int e = lane; e < 2 * C::NPIECE; e += 32) {
           const int kvsel = e >= C::NPIECE, pc = e % C::NPIECE;
           const uint4 val = reinterpret_cast<const uint4 *>(
@@ -572,10 +581,11 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
         den += wgt * s.red_l[w][g];
       }
       if (single) {
-        p.out[qrow * D + e] = num / den;
+        p.out[guard(qrow * D + e, 1, (long long)p.L * p.B * p.Hq * D, p.status)] = num / den;
       } else {
-        p.ws_o[(size_t)item * G * D + e] = num;
-        if (e % D == 0) p.ws_ml[(size_t)item * G + g] = make_float2(M, den);
+        const long long wi = guard(item, 1, p.ws_items, p.status);
+        p.ws_o[wi * G * D + e] = num;
+        if (e % D == 0) p.ws_ml[wi * G + g] = make_float2(M, den);
       }
     }
     if (!single) {
@@ -584,24 +594,27 @@ __device__ __forceinline__ void consume(const DecParams &p, DecSmem<Tin, D, G> &
       if (tid == 0) {
         if (!s.init_seen) s.init_seen = wait_init(p, &s.abort_flag);
         // without the counters (a wait gave up) no item combines the group
-        s.last = s.init_seen && atomicAdd(&p.ctrl[kCtrlGroup + f.group], 1) == f.nch - 1;
+        s.last = s.init_seen && atomicAdd(&p.ctrl[guard(kCtrlGroup + f.group, 1, p.n_ctrl,
+                                                        p.status)],
+                                          1) == f.nch - 1;
       }
       named_bar_sync(1, kWarps * 32);
       if (s.last) {
         __threadfence();
+        const long long ib = guard(item_base, f.nch, p.ws_items, p.status);
         for (int e = tid; e < G * D; e += kWarps * 32) {
           const int g = e / D;
           float M = -INFINITY;
           for (int c = 0; c < f.nch; ++c)
-            M = fmaxf(M, __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]).x);
+            M = fmaxf(M, __ldcg(&p.ws_ml[(size_t)(ib + c) * G + g]).x);
           float num = 0.f, den = 0.f;
           for (int c = 0; c < f.nch; ++c) {
-            const float2 ml = __ldcg(&p.ws_ml[(size_t)(item_base + c) * G + g]);
+            const float2 ml = __ldcg(&p.ws_ml[(size_t)(ib + c) * G + g]);
             const float wgt = fast_exp2(ml.x - M);
             den += wgt * ml.y;
-            num += wgt * __ldcg(&p.ws_o[(size_t)(item_base + c) * G * D + e]);
+            num += wgt * __ldcg(&p.ws_o[(size_t)(ib + c) * G * D + e]);
           }
-          p.out[qrow * D + e] = num / den;
+          p.out[guard(qrow * D + e, 1, (long long)p.L * p.B * p.Hq * D, p.status)] = num / den;
         }
       }
     }
@@ -632,7 +645,9 @@ __device__ __forceinline__ void prefetch_first_item(const DecParams &p) {
     const int r0 = chunk * p.item_rows, r1 = min(len, r0 + p.item_rows);
     const int rows = min(r1 - r0, C::STAGES * C::CR);
     if (rows <= 0) return;
-    const size_t off = ((size_t)unit * p.cap[l] + r0) * C::ROW_BYTES;
+    const size_t off = guard((long long)unit * p.cap[l] + r0, rows, (long long)units * p.cap[l],
+                             p.status) *
+                       C::ROW_BYTES;
     bulk_prefetch_l2((const uint8_t *)p.kc[l] + off, (uint32_t)rows * C::ROW_BYTES);
     bulk_prefetch_l2((const uint8_t *)p.vc[l] + off, (uint32_t)rows * C::ROW_BYTES);
     return;
@@ -834,6 +849,8 @@ size_t plan(const ripple_decode_desc *d, const int32_t *caps, void *ws, DecParam
   if (p != nullptr) {
     uint8_t *base = (uint8_t *)ws;
     p->item_rows = rows;
+    p->ws_items = (long long)items;
+    p->n_ctrl = (int)(kCtrlGroup + groups);
     p->ctrl = (int *)base;
     p->ws_ml = (float2 *)(base + ctrl);
     p->ws_o = (float *)(base + ctrl + ml);

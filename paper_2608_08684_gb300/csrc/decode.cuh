@@ -23,6 +23,8 @@ struct DecParams {
                     // counters are zeroed
   long long wait_cycles;  // bound of the in-kernel waits
   int item_rows;          // cache rows per work item
+  long long ws_items;     // work items the partials (ws_o, ws_ml) have room for
+  int n_ctrl;             // words of the control block
   const void *kc[RIPPLE_MAX_LAYERS];
   const void *vc[RIPPLE_MAX_LAYERS];
   int cap[RIPPLE_MAX_LAYERS];

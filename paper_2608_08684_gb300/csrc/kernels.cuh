@@ -45,7 +45,8 @@ CompressWs carve_compress_ws(const LayerGeom &g, void *base);
 
 // Scoring, SIMT fp32 path (any dtype).
 cudaError_t launch_score_simt(const LayerGeom &g, const void *q_win, const void *k,
-                              const CompressWs &ws, float *votes, cudaStream_t st);
+                              const CompressWs &ws, float *votes, int32_t *status,
+                              cudaStream_t st);
 // Scoring, tcgen05 tensor-core path (bf16, d = 128).
 bool score_tc_supported(const LayerGeom &g);
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
@@ -62,7 +63,7 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
 // writes idx[l] [units][n_keep[l]].
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
                           const CompressWs &ws, const int *n_keep, int32_t *const *idx,
-                          cudaStream_t st);
+                          int32_t *status, cudaStream_t st);
 // idx = 0..T-1 for every unit (keep-all case).
 cudaError_t launch_iota(const LayerGeom &g, int32_t *idx, cudaStream_t st);
 // Gather kept K and V rows of n_layers layers into [units][cap[l]][d].

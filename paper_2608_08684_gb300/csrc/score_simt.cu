@@ -77,7 +77,8 @@ __device__ __forceinline__ void combine(float &m, float &l, float m2, float l2) 
 
 template <typename Tin, int D>
 __global__ void __launch_bounds__(kThreads) score_pass1_simt(LayerGeom g, const Tin *q_win,
-                                                             const Tin *k, float2 *partial) {
+                                                             const Tin *k, float2 *partial,
+                                                             int32_t *status) {
   extern __shared__ float smem[];
   float *Ks = smem;
   float *Qs = smem + kScoreChunk * (D + 1);
@@ -117,11 +118,14 @@ __global__ void __launch_bounds__(kThreads) score_pass1_simt(LayerGeom g, const 
       const float l2 = __shfl_xor_sync(0xffffffffu, l, o);
       combine(m, l, m2, l2);
     }
-    if (tk == 0 && r < g.R) partial[((size_t)unit * n_chunks + chunk) * g.R + r] = make_float2(m, l);
+    if (tk == 0 && r < g.R)
+      partial[guard(((long long)unit * n_chunks + chunk) * g.R + r, 1,
+                    (long long)g.units * n_chunks * g.R, status)] = make_float2(m, l);
   }
 }
 
-__global__ void merge_row_stats(LayerGeom g, int n_chunks, const float2 *partial, float *lognorm) {
+__global__ void merge_row_stats(LayerGeom g, int n_chunks, const float2 *partial, float *lognorm,
+                                int32_t *status) {
   const int unit = blockIdx.x;
   for (int r = threadIdx.x; r < g.R; r += blockDim.x) {
     float m = -INFINITY, l = 0.f;
@@ -129,14 +133,14 @@ __global__ void merge_row_stats(LayerGeom g, int n_chunks, const float2 *partial
       const float2 p = partial[((size_t)unit * n_chunks + c) * g.R + r];
       combine(m, l, p.x, p.y);
     }
-    lognorm[(size_t)unit * g.R + r] = m + log2f(l);
+    lognorm[guard((long long)unit * g.R + r, 1, (long long)g.units * g.R, status)] = m + log2f(l);
   }
 }
 
 template <typename Tin, int D>
 __global__ void __launch_bounds__(kThreads) score_pass2_simt(LayerGeom g, const Tin *q_win,
                                                              const Tin *k, const float *lognorm,
-                                                             float *votes) {
+                                                             float *votes, int32_t *status) {
   extern __shared__ float smem[];
   float *Ks = smem;
   float *Qs = smem + kScoreChunk * (D + 1);
@@ -173,13 +177,13 @@ __global__ void __launch_bounds__(kThreads) score_pass2_simt(LayerGeom g, const 
     const int t = key0 + threadIdx.x;
     float s = 0.f;
     for (int i = 0; i < kRowsPerGroup; ++i) s += red[i * (kScoreChunk + 1) + threadIdx.x];
-    if (t < g.P) votes[(size_t)unit * g.P + t] = s;
+    if (t < g.P) votes[guard((long long)unit * g.P + t, 1, (long long)g.units * g.P, status)] = s;
   }
 }
 
 template <typename Tin, int D>
 cudaError_t launch_typed(const LayerGeom &g, const void *q_win, const void *k,
-                         const CompressWs &ws, float *votes, cudaStream_t st) {
+                         const CompressWs &ws, float *votes, int32_t *status, cudaStream_t st) {
   const size_t smem1 = sizeof(float) * (kScoreChunk + kRowsPerGroup) * (D + 1);
   const size_t smem2 = smem1 + sizeof(float) * kRowsPerGroup * (kScoreChunk + 1);
   cudaError_t e;
@@ -191,12 +195,12 @@ cudaError_t launch_typed(const LayerGeom &g, const void *q_win, const void *k,
   if (e != cudaSuccess) return e;
   const int n_chunks = (g.T + kScoreChunk - 1) / kScoreChunk;
   score_pass1_simt<Tin, D><<<dim3(n_chunks, g.units), kThreads, smem1, st>>>(
-      g, (const Tin *)q_win, (const Tin *)k, ws.row_partial);
-  merge_row_stats<<<g.units, 256, 0, st>>>(g, n_chunks, ws.row_partial, ws.row_lognorm);
+      g, (const Tin *)q_win, (const Tin *)k, ws.row_partial, status);
+  merge_row_stats<<<g.units, 256, 0, st>>>(g, n_chunks, ws.row_partial, ws.row_lognorm, status);
   const int n_chunks2 = (g.P + kScoreChunk - 1) / kScoreChunk;
   if (n_chunks2 > 0)
     score_pass2_simt<Tin, D><<<dim3(n_chunks2, g.units), kThreads, smem2, st>>>(
-        g, (const Tin *)q_win, (const Tin *)k, ws.row_lognorm, votes);
+        g, (const Tin *)q_win, (const Tin *)k, ws.row_lognorm, votes, status);
   count_launches(n_chunks2 > 0 ? 3 : 2);
   return cudaGetLastError();
 }
@@ -204,13 +208,14 @@ cudaError_t launch_typed(const LayerGeom &g, const void *q_win, const void *k,
 }  // namespace
 
 cudaError_t launch_score_simt(const LayerGeom &g, const void *q_win, const void *k,
-                              const CompressWs &ws, float *votes, cudaStream_t st) {
+                              const CompressWs &ws, float *votes, int32_t *status,
+                              cudaStream_t st) {
   if (g.dtype == RIPPLE_F32) {
-    if (g.D == 64) return launch_typed<float, 64>(g, q_win, k, ws, votes, st);
-    return launch_typed<float, 128>(g, q_win, k, ws, votes, st);
+    if (g.D == 64) return launch_typed<float, 64>(g, q_win, k, ws, votes, status, st);
+    return launch_typed<float, 128>(g, q_win, k, ws, votes, status, st);
   }
-  if (g.D == 64) return launch_typed<__nv_bfloat16, 64>(g, q_win, k, ws, votes, st);
-  return launch_typed<__nv_bfloat16, 128>(g, q_win, k, ws, votes, st);
+  if (g.D == 64) return launch_typed<__nv_bfloat16, 64>(g, q_win, k, ws, votes, status, st);
+  return launch_typed<__nv_bfloat16, 128>(g, q_win, k, ws, votes, status, st);
 }
 
 }  // namespace ripple

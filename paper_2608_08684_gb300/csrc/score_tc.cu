@@ -332,7 +332,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!warp_wait(&ms->pub_full[slot], (k / kPubSlots) & 1, ms, p.status)) break;
       const ItemRef it = item_of(p, k);
       // One partial per item: the two warpgroups' statistics combined here.
-      float2 *mine = p.partial + ((size_t)it.unit * p.n_ch + it.chunk) * C::R;
+      float2 *mine = p.partial + guard((long long)it.unit * p.n_ch + it.chunk, 1,
+                                       (long long)p.units * p.n_ch, p.status) *
+                                     C::R;
 #pragma unroll
       for (int j = 0; j < RJ; ++j) {
         const int r = lane + 32 * j;
@@ -346,13 +348,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) {
         mbar_arrive(&ms->pub_empty[slot]);
         __threadfence();  // the item's partial becomes visible GPU-wide before it is counted
-        last = atomicAdd(&p.ctrl[it.unit], 1) == p.n_ch - 1;
+        last = atomicAdd(&p.ctrl[guard(it.unit, 1, p.units, p.status)], 1) == p.n_ch - 1;
       }
       last = __shfl_sync(0xffffffffu, last, 0);
       if (last) {
         // Last item of the unit: merge its n_ch partials per row.
         __threadfence();
-        const float2 *part = p.partial + (size_t)it.unit * p.n_ch * C::R;
+        const float2 *part =
+            p.partial + guard((long long)it.unit * p.n_ch, p.n_ch, (long long)p.units * p.n_ch,
+                              p.status) *
+                            C::R;
         float mm[RJ], ll[RJ];
 #pragma unroll
         for (int j = 0; j < RJ; ++j) {
@@ -374,10 +379,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 #pragma unroll
         for (int j = 0; j < RJ; ++j)
-          p.lognorm[(size_t)it.unit * C::R + lane + 32 * j] = mm[j] + __log2f(ll[j]);
+          p.lognorm[guard(it.unit, 1, p.units, p.status) * C::R + lane + 32 * j] =
+              mm[j] + __log2f(ll[j]);
         __threadfence();
         __syncwarp();
-        if (lane == 0) st_release(&p.ctrl[p.units + it.unit], 1);
+        if (lane == 0) st_release(&p.ctrl[guard(p.units + it.unit, 1, 2LL * p.units, p.status)], 1);
       }
     }
   } else {
@@ -478,10 +484,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         int t0, t1;
         tiles_of(p, it, 2, t0, t1);
         if (t1 > t0) {
-          if (wtid == 0) wait_ready(&p.ctrl[p.units + it.unit], ms, p.status);
+          if (wtid == 0)
+            wait_ready(&p.ctrl[guard(p.units + it.unit, 1, 2LL * p.units, p.status)], ms, p.status);
           named_bar_sync(3 + wg, 128);
           for (int r = wtid; r < C::R; r += 128)
-            ms->off[wg][r] = __ldcg(&p.lognorm[(size_t)it.unit * C::R + r]);
+            ms->off[wg][r] = __ldcg(&p.lognorm[guard(it.unit, 1, p.units, p.status) * C::R + r]);
           named_bar_sync(3 + wg, 128);
         }
         const float4 *off4 = (const float4 *)ms->off[wg];
@@ -526,7 +533,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float vote = ((vs[0].x + vs[0].y) + (vs[1].x + vs[1].y)) +
                              ((vs[2].x + vs[2].y) + (vs[3].x + vs[3].y));
           const int key = t * kTile + lrow;
-          if (key < p.P) p.votes[(size_t)it.unit * p.P + key] = vote;
+          if (key < p.P)
+            p.votes[guard((long long)it.unit * p.P + key, 1, (long long)p.units * p.P, p.status)] =
+                vote;
         }
       }
     }

@@ -363,7 +363,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int slot = k % kPubSlots;
       if (!warp_wait(&ms->pub_full[slot], (k / kPubSlots) & 1, ms, p.status)) break;
       const ItemRef it = item_of(p, k);
-      float2 *mine = p.partial + ((size_t)it.unit * p.n_ch + it.chunk) * 128;
+      float2 *mine = p.partial + guard((long long)it.unit * p.n_ch + it.chunk, 1,
+                                       (long long)p.units * p.n_ch, p.status) *
+                                     128;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int r = lane + 32 * j;
@@ -377,12 +379,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) {
         mbar_arrive(&ms->pub_empty[slot]);
         __threadfence();
-        last = atomicAdd(&p.ctrl[it.unit], 1) == p.n_ch - 1;
+        last = atomicAdd(&p.ctrl[guard(it.unit, 1, p.units, p.status)], 1) == p.n_ch - 1;
       }
       last = __shfl_sync(0xffffffffu, last, 0);
       if (last) {
         __threadfence();
-        const float2 *part = p.partial + (size_t)it.unit * p.n_ch * 128;
+        const float2 *part =
+            p.partial + guard((long long)it.unit * p.n_ch, p.n_ch, (long long)p.units * p.n_ch,
+                              p.status) *
+                            128;
         float mm[4], ll[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
@@ -404,10 +409,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-          p.lognorm[(size_t)it.unit * 128 + lane + 32 * j] = mm[j] + __log2f(ll[j]);
+          p.lognorm[guard(it.unit, 1, p.units, p.status) * 128 + lane + 32 * j] =
+              mm[j] + __log2f(ll[j]);
         __threadfence();
         __syncwarp();
-        if (lane == 0) st_release(&p.ctrl[p.units + it.unit], 1);
+        if (lane == 0) st_release(&p.ctrl[guard(p.units + it.unit, 1, 2LL * p.units, p.status)], 1);
       }
     }
   } else {
@@ -496,9 +502,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           // ---------------- a pass-2 tile of item k - kLag: votes of its keys
           // (D[key][row]: this thread's TMEM lane is key t * 128 + r)
           if (s == 0) {
-            if (wtid == 0) wait_ready(&p.ctrl[p.units + st.u2], ms, p.status);
+            if (wtid == 0)
+              wait_ready(&p.ctrl[guard(p.units + st.u2, 1, 2LL * p.units, p.status)], ms,
+                         p.status);
             named_bar_sync(3 + wg, 128);
-            ms->offs[wg][wtid] = __ldcg(&p.lognorm[(size_t)st.u2 * 128 + wtid]);
+            ms->offs[wg][wtid] =
+                __ldcg(&p.lognorm[guard(st.u2, 1, p.units, p.status) * 128 + wtid]);
             named_bar_sync(3 + wg, 128);
           }
           const int t = st.b0 + s;
@@ -539,7 +548,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float vote = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
                                ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
             const int key = t * kTile + r;
-            if (key < p.P) p.votes[(size_t)st.u2 * p.P + key] = vote;
+            if (key < p.P)
+              p.votes[guard((long long)st.u2 * p.P + key, 1, (long long)p.units * p.P, p.status)] =
+                  vote;
           }
         }
       }

@@ -67,7 +67,8 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int *warp_tot, int *t
 
 __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const float *votes,
                                                           uint32_t *keys_global, int n_keep,
-                                                          int in_smem, int32_t *idx) {
+                                                          int in_smem, int32_t *idx,
+                                                          int32_t *status) {
   extern __shared__ uint32_t sm[];
   uint32_t *hist = sm;                              // [kBins]
   int *warp_tot = (int *)(sm + kBins);              // [33]
@@ -209,7 +210,7 @@ __global__ void __launch_bounds__(kThreads) select_kernel(LayerGeom g, const flo
     const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
     const int g_rank = gt_before + __popc(bg & below);
     const int e_rank = eq_before + __popc(be & below);
-    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = t;
+    if (gt || (eq && e_rank < take_eq)) out[guard(g_rank + min(e_rank, take_eq), 1, K, status)] = t;
     gt_before += __popc(bg);
     eq_before += __popc(be);
   }
@@ -292,6 +293,7 @@ struct SelTable {
   int upl;
   int n_keep[kCompressMaxLayers];
   int32_t *idx[kCompressMaxLayers];
+  int32_t *status;
 };
 
 __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
@@ -488,7 +490,8 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
     const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
     const int g_rank = gt_before + __popc(bg & below);
     const int e_rank = eq_before + __popc(be & below);
-    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = k0 + t;
+    if (gt || (eq && e_rank < take_eq))
+      out[guard(g_rank + min(e_rank, take_eq), 1, K, tab.status)] = k0 + t;
     gt_before += __popc(bg);
     eq_before += __popc(be);
   }
@@ -671,7 +674,8 @@ __global__ void __launch_bounds__(kUThreads, 1)
     const int off = cnt[i * kUWarps + wid];
     const int g_rank = (off >> 16) + __popc(bg & below);
     const int e_rank = (off & 0xffff) + __popc(be & below);
-    if (gt || (eq && e_rank < take_eq)) out[g_rank + min(e_rank, take_eq)] = j;
+    if (gt || (eq && e_rank < take_eq))
+      out[guard(g_rank + min(e_rank, take_eq), 1, K, tab.status)] = j;
   }
 }
 
@@ -679,13 +683,14 @@ __global__ void __launch_bounds__(kUThreads, 1)
 
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
                           const CompressWs &ws, const int *n_keep, int32_t *const *idx,
-                          cudaStream_t st) {
+                          int32_t *status, cudaStream_t st) {
   if (n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorInvalidValue;
   // One CTA per unit once the launch has enough units to fill the GPU;
   // fewer units (a single layer) are spread over 8-CTA clusters instead.
   if (g.P <= kUMaxP && (long long)g.units * n_layers >= kUMinUnits) {
     SelTable tab;
     tab.upl = g.units;
+    tab.status = status;
     for (int l = 0; l < n_layers; ++l) {
       tab.n_keep[l] = n_keep[l];
       tab.idx[l] = idx[l];
@@ -702,6 +707,7 @@ cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
   if (per_cta <= kCMaxKeys && (long long)g.units * n_layers * kCluster <= 0x7fffffff) {
     SelTable tab;
     tab.upl = g.units;
+    tab.status = status;
     for (int l = 0; l < n_layers; ++l) {
       tab.n_keep[l] = n_keep[l];
       tab.idx[l] = idx[l];
@@ -723,7 +729,7 @@ cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
   if (e != cudaSuccess) return e;
   for (int l = 0; l < n_layers; ++l) {
     select_kernel<<<g.units, kThreads, smem, st>>>(g, votes + (size_t)l * g.units * g.P, ws.keys,
-                                                   n_keep[l], in_smem, idx[l]);
+                                                   n_keep[l], in_smem, idx[l], status);
     count_launches(1);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;

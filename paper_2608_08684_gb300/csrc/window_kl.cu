@@ -142,16 +142,6 @@ __device__ __forceinline__ float2 g_over_x2(float2 x) {
   return __ffma2_rn(x, h, make_float2(0.5f, 0.5f));
 }
 
-// exp(x) - 1 in fp32: x + x^2 (g(x) / x^2) for |x| <= kKlPolyBound (relative
-// error near 1e-7), else from the exponential.
-__device__ __forceinline__ float expm1_kl(float x) {
-  if (fabsf(x) <= kKlPolyBound) {
-    const float h = g_over_x2(make_float2(x, x)).x;
-    return __fmaf_rn(__fmul_rn(x, x), h, x);
-  }
-  return __fsub_rn(fast_exp2(__fmul_rn(x, kLog2e)), 1.f);
-}
-
 // log1p(t) - t without cancellation: with s = t / (2 + t), log1p(t) =
 // 2 atanh(s) and 2 s - t = -t s, so
 //   log1p(t) - t = -t s + 2 s^3 (1/3 + s^2/5 + s^4/7 + ... + s^10/13);
@@ -480,7 +470,9 @@ __device__ __forceinline__ void kl_produce(const KlParams &P, KlSmem &s, long lo
       if (!kl_wait(&s.p_empty[ps], ((pc >> 1) & 1) ^ 1, &s.abort_flag, P.status, P.wait_cycles))
         break;
       mbar_arrive_expect_tx(&s.p_full[ps], bytes);
-      bulk_g2s(s.p[ps], p + (size_t)it.pos * P.vocab + begin, bytes, &s.p_full[ps]);
+      const long long po = guard((long long)it.pos * P.vocab + begin, bytes / sizeof(Tl),
+                                 (long long)P.n_pos * P.vocab, P.status);
+      bulk_g2s(s.p[ps], p + po, bytes, &s.p_full[ps]);
       ++pc;
     }
     const int st = qc % kKlStages;
@@ -488,8 +480,10 @@ __device__ __forceinline__ void kl_produce(const KlParams &P, KlSmem &s, long lo
                  P.wait_cycles))
       break;
     mbar_arrive_expect_tx(&s.q_full[st], bytes);
-    bulk_g2s(s.q[st], q + ((size_t)it.set * P.n_pos + it.pos) * P.vocab + begin, bytes,
-             &s.q_full[st]);
+    const long long qo = guard(((long long)it.set * P.n_pos + it.pos) * P.vocab + begin,
+                               bytes / sizeof(Tl), (long long)P.n_sets * P.n_pos * P.vocab,
+                               P.status);
+    bulk_g2s(s.q[st], q + qo, bytes, &s.q_full[st]);
     ++qc;
   }
   // Copies still in flight must land before the CTA exits (after an abort;
@@ -543,8 +537,9 @@ __device__ __forceinline__ void kl_consume(const KlParams &P, KlSmem &s, int war
     ++qc;
     if (lane == 0) {
       float4 *dst = reinterpret_cast<float4 *>(
-          P.part + ((size_t)it.set * P.n_pos + it.pos) * n_parts + it.slice * kKlConsumerWarps +
-          warp);
+          P.part + guard(((long long)it.set * P.n_pos + it.pos) * n_parts +
+                             it.slice * kKlConsumerWarps + warp,
+                         1, (long long)P.n_sets * P.n_pos * n_parts, P.status));
       dst[0] = make_float4(r.mp, r.zp, r.c, r.a);
       dst[1] = make_float4(r.b, r.r, __int_as_float(r.kind), 0.f);
     }
@@ -599,20 +594,23 @@ __global__ void __launch_bounds__(kKlMergeWarps * 32)
   if (row >= P.n_sets * P.n_pos) return;
   const int set = row / P.n_pos;
   const int n_parts = P.n_slices * kKlConsumerWarps;
-  const double kl = merge_row<kCached>(P.part + (size_t)row * n_parts, n_parts, lane);
+  const long long rows = (long long)P.n_sets * P.n_pos;
+  const double kl = merge_row<kCached>(
+      P.part + guard((long long)row * n_parts, n_parts, rows * n_parts, P.status), n_parts, lane);
   int old = 0;
   if (lane == 0) {
-    P.row_kl[row] = kl;
-    if (P.kl_out != nullptr) P.kl_out[row] = (float)kl;
+    P.row_kl[guard(row, 1, rows, P.status)] = kl;
+    if (P.kl_out != nullptr) P.kl_out[guard(row, 1, rows, P.status)] = (float)kl;
     __threadfence();
-    old = atomicAdd(&P.set_count[set], 1);
+    old = atomicAdd(&P.set_count[guard(set, 1, P.n_sets, P.status)], 1);
   }
   if (__shfl_sync(0xffffffffu, old, 0) != P.n_pos - 1) return;
   __threadfence();
   double s = 0.0;
-  for (int t = lane; t < P.n_pos; t += 32) s += __ldcg(&P.row_kl[(size_t)set * P.n_pos + t]);
+  const long long r0 = guard((long long)set * P.n_pos, P.n_pos, rows, P.status);
+  for (int t = lane; t < P.n_pos; t += 32) s += __ldcg(&P.row_kl[r0 + t]);
   s = warp_sum_d(s);
-  if (lane == 0) P.d_out[set] = (float)(s / (double)P.n_pos);
+  if (lane == 0) P.d_out[guard(set, 1, P.n_sets, P.status)] = (float)(s / (double)P.n_pos);
 }
 
 // ------------------------------------------------------------ host side

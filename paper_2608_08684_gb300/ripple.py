@@ -13,9 +13,13 @@ import os
 
 import torch
 
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libripple.so")
+# RIPPLE_CHECKED=1 selects the bounds-checked build of the same library.
+CHECKED = os.environ.get("RIPPLE_CHECKED", "0") == "1"
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                        "libripple_checked.so" if CHECKED else "libripple.so")
 if not os.path.exists(LIB_PATH):
-    raise ImportError(f"{LIB_PATH} is not built: call paper_2608_08684_gb300.build.build_library()")
+    raise ImportError(f"{LIB_PATH} is not built: call paper_2608_08684_gb300.build."
+                      f"build_library(checked={CHECKED})")
 _lib = ctypes.CDLL(LIB_PATH)
 
 F32, BF16 = 0, 1

@@ -103,7 +103,9 @@ def test_decode_times_out_then_recovers(lib):
     wl = synth.WORKLOADS["tiny"].replace(n_layers=2, batch=2, n_q_heads=8, n_kv_heads=2,
                                          head_dim=128, dtype="bf16", kv_dist="scaled_sinks",
                                          seed=61)
-    lens0 = [5000, 300]
+    # long caches: many sub-chunk stages per work item, so that stage waits
+    # depend on the other role's progress
+    lens0 = [24000, 9000]
     caps = [n + 2 for n in lens0]
     desc = lib.decode_desc(2, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.torch_dtype)
     ws = torch.empty(lib.ripple_decode_workspace_bytes(desc, caps), dtype=torch.uint8,
@@ -120,10 +122,18 @@ def test_decode_times_out_then_recovers(lib):
         return status, out, kc, vc
 
     torch.cuda.synchronize()
-    with _ShortWaits(lib):
-        status, *_ = run()
-    assert _timed_sync() < 10.0
-    assert int(status.item()) == lib.ETIMEOUT
+    # Whether a wait outlasts the bound depends on timing (an mbarrier wait is
+    # suspended in hardware and may return only when its phase completes), so
+    # the short-bound call is repeated until one of its waits gives up.
+    seen = []
+    for _ in range(5):
+        with _ShortWaits(lib):
+            status, *_ = run()
+        assert _timed_sync() < 10.0
+        seen.append(int(status.item()))
+        if seen[-1] == lib.ETIMEOUT:
+            break
+    assert seen[-1] == lib.ETIMEOUT and set(seen) <= {0, lib.ETIMEOUT}, seen
     # the same workspace (left as the timed-out call left it), default limit
     status, out, kc, vc = run()
     torch.cuda.synchronize()
