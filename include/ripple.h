@@ -207,6 +207,47 @@ ripple_status ripple_compress_layers(const ripple_layer_desc *desc, int32_t n_la
                                      int32_t *n_keep_host, void *workspace,
                                      size_t workspace_bytes, int32_t *dev_status, void *stream);
 
+/* Device workspace bytes ripple_compress_layers_attn needs for n_layers layers
+ * of this shape (RIPPLE_EINVAL for shapes it does not take). */
+ripple_status ripple_compress_layers_attn_workspace_bytes(const ripple_layer_desc *desc,
+                                                          int32_t n_layers, size_t *bytes_host);
+
+/*
+ * ripple_compress_layers_attn -- ripple_compress_layers whose scoring pass also
+ * gives the prefill attention output of the observation-window rows: the
+ * SnapKV scoring that RippleKV keeps (Sec. 4.4, last paragraph; Sec. 2) fused
+ * into the prefill attention of those rows, so that a real prefill reads each
+ * layer's keys once for both (the rows' logits and normalisers are the same
+ * quantities; no paper counterpart beyond that identity).
+ *
+ * For every layer l, batch b, query head q (KV head q / G) and window position
+ * i (token P + i, P = T - w), with the causal mask of the window:
+ *   o_win[l][b][q][i] = sum over t <= P + i of
+ *                       softmax_t(scale * q_win[b][q][i] . k[b][q/G][t]) * v[b][q/G][t]
+ * computed from the same logits and row normalisers as the votes.
+ *
+ * Shapes: bf16, head_dim 128, G * w = 128 window rows (the tensor-core path);
+ * others return RIPPLE_EINVAL.
+ * o_win_host  host array of n_layers device pointers, each fp32
+ *             [B][Hq][w][head_dim], 16-byte aligned, written
+ * workspace   at least ripple_compress_layers_attn_workspace_bytes bytes,
+ *             256-byte aligned, no initialisation needed
+ * Other arguments, outputs and errors as ripple_compress_layers; the kept
+ * counts, indices and gathered rows equal that call's bit for bit. o_win is
+ * accumulated in fp32 from bf16 probabilities (the tensor cores' operand
+ * type) in a fixed order: the same on every run. The call may be captured in a
+ * CUDA graph.
+ */
+ripple_status ripple_compress_layers_attn(const ripple_layer_desc *desc, int32_t n_layers,
+                                          const int64_t *budgets_host,
+                                          const void *const *q_win_host,
+                                          const void *const *k_host, const void *const *v_host,
+                                          void *const *k_out_host, void *const *v_out_host,
+                                          const int32_t *caps_host, int32_t *const *idx_out_host,
+                                          int32_t *n_keep_host, float *const *o_win_host,
+                                          void *workspace, size_t workspace_bytes,
+                                          int32_t *dev_status, void *stream);
+
 /*
  * ripple_select_layer -- steps 2-4 of ripple_compress_layer (pooling, top-k
  * selection with the window appended, gather) from caller-provided votes

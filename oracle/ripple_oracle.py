@@ -177,6 +177,27 @@ def window_votes(q_win, k, scale):
     return probs.sum(axis=0), row_max, row_sum
 
 
+def window_attention(q_win, k, v, scale):
+    """Prefill attention output of the observation-window rows of one unit
+    (the rows whose softmax SnapKV's scoring reads, reading R5; computed here
+    directly from that definition, with the same causal mask).
+
+    q_win: [G][w][d]; k, v: [T][d]. Returns [G][w][d] float64: row (g, i), at
+    token P + i, is sum over keys t <= P + i of softmax_t(scale q . k_t) v_t.
+    """
+    G, w, d = q_win.shape
+    T = k.shape[0]
+    P = T - w
+    out = np.zeros((G, w, v.shape[1]))
+    for g in range(G):
+        for i in range(w):
+            vis = P + i + 1
+            logits = (k[:vis] @ q_win[g, i]) * scale
+            e = np.exp(logits - logits.max())
+            out[g, i] = (e / e.sum()) @ v[:vis]
+    return out
+
+
 def pool_scores(votes, kernel, kind="max"):
     """1-D pooling of the prefix votes (reading R6), in the dtype of `votes`.
 

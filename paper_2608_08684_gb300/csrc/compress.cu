@@ -172,27 +172,54 @@ static CompressWs carve_layers_ws(const LayerGeom &g, int n_layers, void *base) 
   return carve_compress_ws(all, base);
 }
 
+// The multi-layer workspace with the window rows' output partials after it.
+static CompressWs carve_layers_attn_ws(const LayerGeom &g, int n_layers, void *base) {
+  CompressWs w = carve_layers_ws(g, n_layers, base);
+  uint8_t *p = (uint8_t *)base;
+  size_t off = w.bytes;
+  const size_t units = (size_t)g.units * n_layers;
+  w.o_part = p ? (float *)(p + off) : nullptr;
+  off += round_up(sizeof(float) * units * score_tc1_max_items(g) * g.R * g.D);
+  w.o_count = p ? (int32_t *)(p + off) : nullptr;
+  off += round_up(sizeof(int32_t) * units);
+  w.bytes = off;
+  return w;
+}
+
+static bool layers_geom(const ripple_layer_desc *desc, int32_t n_layers, LayerGeom *g) {
+  return make_geom(desc, g) && n_layers >= 1 && n_layers <= RIPPLE_COMPRESS_MAX_LAYERS &&
+         (int64_t)g->units * n_layers <= 65535;
+}
+
 extern "C" ripple_status ripple_compress_layers_workspace_bytes(const ripple_layer_desc *desc,
                                                                 int32_t n_layers,
                                                                 size_t *bytes_host) {
   LayerGeom g;
-  if (!make_geom(desc, &g) || bytes_host == nullptr || n_layers < 1 ||
-      n_layers > RIPPLE_COMPRESS_MAX_LAYERS || (int64_t)g.units * n_layers > 65535)
-    return RIPPLE_EINVAL;
+  if (!layers_geom(desc, n_layers, &g) || bytes_host == nullptr) return RIPPLE_EINVAL;
   *bytes_host = carve_layers_ws(g, n_layers, nullptr).bytes;
   return RIPPLE_OK;
 }
 
-extern "C" ripple_status ripple_compress_layers(
+extern "C" ripple_status ripple_compress_layers_attn_workspace_bytes(const ripple_layer_desc *desc,
+                                                                     int32_t n_layers,
+                                                                     size_t *bytes_host) {
+  LayerGeom g;
+  if (!layers_geom(desc, n_layers, &g) || bytes_host == nullptr || !score_tc1_supported(g))
+    return RIPPLE_EINVAL;
+  *bytes_host = carve_layers_attn_ws(g, n_layers, nullptr).bytes;
+  return RIPPLE_OK;
+}
+
+// Both multi-layer entry points; with o_win_host (non-NULL) the scoring pass
+// also gives the window rows' attention output of every layer.
+static ripple_status compress_layers_impl(
     const ripple_layer_desc *desc, int32_t n_layers, const int64_t *budgets_host,
     const void *const *q_win_host, const void *const *k_host, const void *const *v_host,
     void *const *k_out_host, void *const *v_out_host, const int32_t *caps_host,
-    int32_t *const *idx_out_host, int32_t *n_keep_host, void *workspace, size_t workspace_bytes,
-    int32_t *dev_status, void *stream) {
+    int32_t *const *idx_out_host, int32_t *n_keep_host, float *const *o_win_host,
+    void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
   LayerGeom g;
-  if (!make_geom(desc, &g) || n_layers < 1 || n_layers > RIPPLE_COMPRESS_MAX_LAYERS ||
-      (int64_t)g.units * n_layers > 65535)
-    return RIPPLE_EINVAL;
+  if (!layers_geom(desc, n_layers, &g)) return RIPPLE_EINVAL;
   if (!budgets_host || !q_win_host || !k_host || !v_host || !k_out_host || !v_out_host ||
       !caps_host || !idx_out_host || !n_keep_host || !workspace || ((uintptr_t)workspace & 255u))
     return RIPPLE_EINVAL;
@@ -202,19 +229,21 @@ extern "C" ripple_status ripple_compress_layers(
   for (int l = 0; l < n_layers; ++l) {
     if (budgets_host[l] < 0 || !aligned(q_win_host[l]) || !aligned(k_host[l]) ||
         !aligned(v_host[l]) || !aligned(k_out_host[l]) || !aligned(v_out_host[l]) ||
-        !aligned(idx_out_host[l]))
+        !aligned(idx_out_host[l]) || (o_win_host != nullptr && !aligned(o_win_host[l])))
       return RIPPLE_EINVAL;
     n[l] = ripple_keep_count(budgets_host[l], g.T, g.W);
     cap[l] = caps_host[l];
     if (n[l] < 0 || cap[l] < n[l]) return RIPPLE_EINVAL;
   }
-  const CompressWs ws = carve_layers_ws(g, n_layers, workspace);
+  if (o_win_host != nullptr && !score_tc1_supported(g)) return RIPPLE_EINVAL;
+  const CompressWs ws = o_win_host ? carve_layers_attn_ws(g, n_layers, workspace)
+                                   : carve_layers_ws(g, n_layers, workspace);
   if (workspace_bytes < ws.bytes) return RIPPLE_EWORKSPACE;
   cudaStream_t st = (cudaStream_t)stream;
   if (g.P > 0 && score_tc1_supported(g)) {
     // All layers in three launches: scoring, selection, gather.
     RIPPLE_CUDA_TRY(launch_score_tc1(g, n_layers, q_win_host, k_host, ws, ws.votes, dev_status,
-                                     st));
+                                     st, o_win_host ? v_host : nullptr, o_win_host));
     RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st));
     RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
                                   (const int32_t *const *)idx_out_host, n, k_out_host,
@@ -240,4 +269,27 @@ extern "C" ripple_status ripple_compress_layers(
   }
   for (int l = 0; l < n_layers; ++l) n_keep_host[l] = n[l];
   return RIPPLE_OK;
+}
+
+extern "C" ripple_status ripple_compress_layers(
+    const ripple_layer_desc *desc, int32_t n_layers, const int64_t *budgets_host,
+    const void *const *q_win_host, const void *const *k_host, const void *const *v_host,
+    void *const *k_out_host, void *const *v_out_host, const int32_t *caps_host,
+    int32_t *const *idx_out_host, int32_t *n_keep_host, void *workspace, size_t workspace_bytes,
+    int32_t *dev_status, void *stream) {
+  return compress_layers_impl(desc, n_layers, budgets_host, q_win_host, k_host, v_host,
+                              k_out_host, v_out_host, caps_host, idx_out_host, n_keep_host,
+                              nullptr, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" ripple_status ripple_compress_layers_attn(
+    const ripple_layer_desc *desc, int32_t n_layers, const int64_t *budgets_host,
+    const void *const *q_win_host, const void *const *k_host, const void *const *v_host,
+    void *const *k_out_host, void *const *v_out_host, const int32_t *caps_host,
+    int32_t *const *idx_out_host, int32_t *n_keep_host, float *const *o_win_host,
+    void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
+  if (o_win_host == nullptr) return RIPPLE_EINVAL;
+  return compress_layers_impl(desc, n_layers, budgets_host, q_win_host, k_host, v_host,
+                              k_out_host, v_out_host, caps_host, idx_out_host, n_keep_host,
+                              o_win_host, workspace, workspace_bytes, dev_status, stream);
 }

@@ -39,6 +39,8 @@ struct CompressWs {
   float *votes;         // [units][P] unpooled votes (when scores_out is NULL)
   uint32_t *keys;       // [units][P] pooled-score sort keys (long prefixes only)
   int32_t *counters;    // small control block
+  float *o_part;        // with the window rows' output: [units][items][G*w][d] partials
+  int32_t *o_count;     // with the window rows' output: [units] items written
   size_t bytes;
 };
 CompressWs carve_compress_ws(const LayerGeom &g, void *base);
@@ -52,13 +54,18 @@ bool score_tc_supported(const LayerGeom &g);
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
                             const CompressWs &ws, float *votes, int32_t *status,
                             cudaStream_t st);
-// Scoring with the window queries in TMEM (bf16, d = 128, G * w = 128 rows),
+// Scoring on the tensor cores for G * w = 128 window rows (bf16, d = 128),
 // for n_layers layers of the same shape in one launch; ws is carved for
-// n_layers * g.units units and votes is [n_layers][g.units][P].
+// n_layers * g.units units and votes is [n_layers][g.units][P]. With v (the
+// values of every layer) the same pass also gives the window rows' attention
+// output o_win[l] [B][Hq][w][d] fp32 (ws carved with its partials).
 bool score_tc1_supported(const LayerGeom &g);
 cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const *q_win,
                              const void *const *k, const CompressWs &ws, float *votes,
-                             int32_t *status, cudaStream_t st);
+                             int32_t *status, cudaStream_t st, const void *const *v = nullptr,
+                             float *const *o_win = nullptr);
+// Items per unit of launch_score_tc1 at most (sizes the output partials).
+int score_tc1_max_items(const LayerGeom &g);
 // Pooling + exact top-k per unit of n_layers layers (votes [n_layers][units][P]);
 // writes idx[l] [units][n_keep[l]].
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,

@@ -21,6 +21,18 @@
 // alternate tiles, warp 10 = publisher of pass-1 results. Every wait is
 // bounded; on timeout the CTA raises RIPPLE_ETIMEOUT, every role leaves its
 // loop and TMEM is released.
+//
+// With the window rows' attention output (kO; the scoring fused into the
+// prefill attention of the window rows, so that a real prefill reads the keys
+// for both in one pass): pass 2 covers every key, causal inside the window;
+// the producer streams each value tile behind the next key tile through the
+// same ring (three stages); the epilogue writes the tile's probabilities as
+// bf16 into a shared-memory tile (MN-major, the A operand) and the MMA warp
+// accumulates O[row][dim] += P . V in the last 128 TMEM columns (V, MN-major,
+// the B operand). The probabilities are final (pass 1 has fixed every row's
+// normaliser), so O needs no rescaling. At an item's end both warpgroups
+// write its partial O to the workspace; the item that completes its unit
+// sums the unit's partials in item order into the output.
 #include <cuda.h>
 #include <math.h>
 
@@ -37,20 +49,34 @@ constexpr int kTile = 128;                      // keys per tile
 constexpr int kHalfBytes = kTile * 64 * 2;      // one TMA box: 64 dims of 128 keys
 constexpr int kTileBytes = 2 * kHalfBytes;
 constexpr int kThreads = 352;
-constexpr int kNK = 4;                          // key-tile stages
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
-constexpr int kNA = 4;                          // accumulators in TMEM (128 columns each)
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
-static_assert(kNA * 128 <= 512, "TMEM columns");
+constexpr int kMaxStages = 4;
+
+// With kO (the window rows' attention output as well as the votes) pass 2
+// covers every key and also streams the value tiles, multiplies the
+// probabilities by them on the tensor cores and accumulates O in TMEM; the
+// probabilities go through a 32 KB shared-memory tile, so the ring has one
+// stage less, and O takes the last 128 TMEM columns.
+template <bool kO>
+struct Tc1Cfg {
+  static constexpr int NK = kO ? 3 : 4;   // ring stages (key tiles; value tiles with kO)
+  static constexpr int NA = kO ? 3 : 4;   // S accumulators in TMEM (128 columns each)
+  static constexpr uint32_t OCol = NA * 128;  // O accumulator (kO)
+  static_assert(NA * 128 + (kO ? 128 : 0) <= 512, "TMEM columns");
+  static_assert(NK <= kMaxStages && NA <= kMaxStages, "barrier arrays");
+};
 
 struct Tc1Params {
   int units, upl, T, P, W, Hq, Hkv, G;  // units of all layers, units per layer
-  int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys)
+  int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys; all with kO)
   int tpi, n_ch;           // key tiles per item, items per unit
   int total_items;
   float scale2;
-  const uint8_t *q[kCompressMaxLayers];  // per layer: window queries [B][Hq][W][128] bf16
+  float *o_win[kCompressMaxLayers];  // kO, per layer: window-row outputs [B][Hq][W][128] fp32
+  float *o_part;     // kO: [units][n_ch][128][128] fp32 per-item partial outputs
+  int *o_count;      // kO: [units] items of unit u whose partial is written
   float2 *partial;   // [units][n_ch][128] (max, sum) per item and row, log2 domain
   float *lognorm;    // [units][128]
   float *votes;      // [units][P], layer-major
@@ -124,21 +150,30 @@ __device__ __forceinline__ void seq_at(const Step &s, int j, int &pass, int &idx
 }
 
 struct Misc {
-  uint64_t k_full[kNK], k_empty[kNK], q_full, q_empty, acc_full[kNA], acc_empty[kNA];
+  uint64_t k_full[kMaxStages], k_empty[kMaxStages], q_full, q_empty;
+  uint64_t acc_full[kMaxStages], acc_empty[kMaxStages];
   uint64_t qs_full, qs_empty;           // pass-2 queries in shared memory
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
+  uint64_t p_full, p_empty, o_full, o_empty;  // kO: probability tile, O accumulator
   uint32_t tmem_base;
   int abort_flag;
+  int o_last;                           // kO: this CTA completed its unit's partials
   long long wait_cycles;  // bound of the waits of this launch
   float2 pstat[kPubSlots][2][128];      // pass-1 row statistics per slot and warpgroup
   alignas(16) float offs[2][128];       // per warpgroup: the pass-2 item's row log-normalisers
 };
 
-constexpr int kOffQs = kNK * kTileBytes;          // pass-2 queries: two 64-dim halves
-constexpr int kOffQ1 = kOffQs + kTileBytes;       // pass-1 queries
-constexpr int kOffMisc = kOffQ1 + kTileBytes;
-constexpr int kSmemBytes = kOffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+// Shared memory: the ring, the pass-2 and pass-1 queries (two 64-dim halves
+// each), with kO the probability tile, then the barriers and statistics.
+template <bool kO>
+struct Tc1Smem {
+  static constexpr int OffQs = Tc1Cfg<kO>::NK * kTileBytes;
+  static constexpr int OffQ1 = OffQs + kTileBytes;
+  static constexpr int OffP = OffQ1 + kTileBytes;
+  static constexpr int OffMisc = OffP + (kO ? kTileBytes : 0);
+  static constexpr int Bytes = OffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
+  static_assert(Bytes <= 227 * 1024, "shared memory budget");
+};
 
 __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *ms,
                                          int32_t *status) {
@@ -183,35 +218,91 @@ __device__ __forceinline__ void combine(float &m, float &l, float m2, float l2) 
   m = mm;
 }
 
-// Kernel argument: the keys of every layer as 3-D tensor maps [unit][T][128],
-// the window queries of every layer as 2-D maps [B * Hq * W][128], and the
-// parameters.
+// Kernel argument: the keys (and with kO the values) of every layer as 3-D
+// tensor maps [unit][T][128], the window queries of every layer as 2-D maps
+// [B * Hq * W][128], and the parameters.
 struct Tc1Launch {
   CUtensorMap kmap[kCompressMaxLayers];
   CUtensorMap qmap[kCompressMaxLayers];
+  CUtensorMap vmap[kCompressMaxLayers];
   Tc1Params p;
 };
 
+// With kO the producer and the MMA warp walk a step as: the pass-1 key tiles,
+// then for the pass-2 item key tile s followed by value tile s - 1 (the order
+// the MMA warp consumes them in: it multiplies a tile's probabilities by its
+// values after issuing the next tile's logits), then the last value tile.
+// kind 1: pass-1 key tile, 2: pass-2 key tile, 3: pass-2 value tile.
+__device__ __forceinline__ void oseq_at(const Step &s, int j, int &kind, int &idx) {
+  if (j < s.n1) {
+    kind = 1;
+    idx = j;
+    return;
+  }
+  const int q = j - s.n1;
+  if (q == 0) {
+    kind = 2;
+    idx = 0;
+  } else if (q == 2 * s.n2 - 1) {
+    kind = 3;
+    idx = s.n2 - 1;
+  } else if (q & 1) {
+    kind = 2;
+    idx = (q + 1) >> 1;
+  } else {
+    kind = 3;
+    idx = (q >> 1) - 1;
+  }
+}
+
+// Probabilities of one key (this thread's TMEM lane) for the 128 window rows
+// (fp32 bit patterns, row e in pr[e / 32][e % 32]), as bf16, into the shared-memory tile in the MN-major, 128-byte-swizzled
+// layout the tensor core reads as the A operand of O = P . V: rows 0-63 and
+// 64-127 in two 16 KB halves, in each the key's 128-byte line holds its 64
+// rows, 16-byte chunk c at position c ^ (key mod 8).
+__device__ __forceinline__ void store_p_row(uint8_t *ptile, int key, const uint32_t (&pr)[4][32]) {
+#pragma unroll
+  for (int half = 0; half < 2; ++half)
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      uint32_t w[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int e = half * 64 + c * 8 + 2 * i;  // rows e, e + 1
+        const __nv_bfloat162 b = __floats2bfloat162_rn(__uint_as_float(pr[e >> 5][e & 31]),
+                                                       __uint_as_float(pr[(e + 1) >> 5][(e + 1) & 31]));
+        w[i] = *reinterpret_cast<const uint32_t *>(&b);
+      }
+      uint8_t *dst = ptile + half * kHalfBytes + (key >> 3) * 1024 + (key & 7) * 128 +
+                     ((c ^ (key & 7)) << 4);
+      *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+template <bool kO>
 __global__ void __launch_bounds__(kThreads, 1)
     score_tc1_kernel(const __grid_constant__ Tc1Launch lp) {
+  using C = Tc1Cfg<kO>;
+  using SM = Tc1Smem<kO>;
   const Tc1Params &p = lp.p;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ktiles = smem;
-  uint8_t *qsm = smem + kOffQs;
-  uint8_t *q1m = smem + kOffQ1;
-  Misc *ms = (Misc *)(smem + kOffMisc);
+  uint8_t *qsm = smem + SM::OffQs;
+  uint8_t *q1m = smem + SM::OffQ1;
+  uint8_t *ptile = smem + SM::OffP;
+  Misc *ms = (Misc *)(smem + SM::OffMisc);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n = items_of_cta(p);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kNK; ++i) {
+    for (int i = 0; i < C::NK; ++i) {
       mbar_init(&ms->k_full[i], 1);
       mbar_init(&ms->k_empty[i], 1);
     }
     mbar_init(&ms->q_full, 1);
     mbar_init(&ms->q_empty, 1);
-    for (int i = 0; i < kNA; ++i) {
+    for (int i = 0; i < C::NA; ++i) {
       mbar_init(&ms->acc_full[i], 1);
       mbar_init(&ms->acc_empty[i], 4);
     }
@@ -222,7 +313,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->pub_empty[i], 1);
     }
     mbar_init(&ms->mma_done, 1);
+    mbar_init(&ms->p_full, 4);
+    mbar_init(&ms->p_empty, 1);
+    mbar_init(&ms->o_full, 1);
+    mbar_init(&ms->o_empty, 8);
     ms->abort_flag = 0;
+    ms->o_last = 0;
     ms->wait_cycles = p.wait_cycles;
     fence_mbar_init();
   }
@@ -244,108 +340,148 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
-        for (int j = 0; j < st.len && ok; ++j) {
-          {
-            int pass, s;
+        const int len = kO ? st.n1 + 2 * st.n2 : st.len;
+        for (int j = 0; j < len && ok; ++j) {
+          int pass, s, kind;
+          if (kO) {
+            oseq_at(st, j, kind, s);
+            pass = kind == 1 ? 1 : 2;
+          } else {
             seq_at(st, j, pass, s);
-            if (pass == 1 && s == 0) {
-              // item k's queries into the pass-1 buffer, once the previous
-              // item's pass-1 MMAs have read it
-              if (!wait_bar(&ms->q_empty, (k & 1) ^ 1, ms, p.status)) {
-                ok = false;
-                break;
-              }
-              const int layer = st.u1 / p.upl, local = st.u1 % p.upl;
-              const int b = local / p.Hkv, h = local % p.Hkv;
-              const int qrow0 = (b * p.Hq + h * p.G) * p.W;
-              mbar_arrive_expect_tx(&ms->q_full, kTileBytes);
-              tma_load_2d(q1m, &lp.qmap[layer], 0, qrow0, &ms->q_full);
-              tma_load_2d(q1m + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->q_full);
-            }
-            if (pass == 2 && s == 0) {
-              // the pass-2 item's queries (rows of its unit) into shared memory
-              if (!wait_bar(&ms->qs_empty, (qcount & 1) ^ 1, ms, p.status)) {
-                ok = false;
-                break;
-              }
-              const int layer = st.u2 / p.upl, local = st.u2 % p.upl;
-              const int b = local / p.Hkv, h = local % p.Hkv;
-              const int qrow0 = (b * p.Hq + h * p.G) * p.W;
-              mbar_arrive_expect_tx(&ms->qs_full, kTileBytes);
-              tma_load_2d(qsm, &lp.qmap[layer], 0, qrow0, &ms->qs_full);
-              tma_load_2d(qsm + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->qs_full);
-              ++qcount;
-            }
-            const int unit = pass == 1 ? st.u1 : st.u2;
-            const int tt = pass == 1 ? st.a0 + s : st.b0 + s;
-            const int ks = kcount % kNK;
-            if (!wait_bar(&ms->k_empty[ks], ((kcount / kNK) & 1) ^ 1, ms, p.status)) {
+            kind = pass;
+          }
+          if (kind == 1 && s == 0) {
+            // item k's queries into the pass-1 buffer, once the previous
+            // item's pass-1 MMAs have read it
+            if (!wait_bar(&ms->q_empty, (k & 1) ^ 1, ms, p.status)) {
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
-            uint8_t *kb = ktiles + ks * kTileBytes;
-            const uint64_t pol = pass == 1 ? keep : drop;
-            const CUtensorMap *km = &lp.kmap[unit / p.upl];
-            const int local = unit % p.upl;
-            tma_load_3d(kb, km, 0, tt * kTile, local, &ms->k_full[ks], pol);
-            tma_load_3d(kb + kHalfBytes, km, 64, tt * kTile, local, &ms->k_full[ks], pol);
-            ++kcount;
+            const int layer = st.u1 / p.upl, local = st.u1 % p.upl;
+            const int b = local / p.Hkv, h = local % p.Hkv;
+            const int qrow0 = (b * p.Hq + h * p.G) * p.W;
+            mbar_arrive_expect_tx(&ms->q_full, kTileBytes);
+            tma_load_2d(q1m, &lp.qmap[layer], 0, qrow0, &ms->q_full);
+            tma_load_2d(q1m + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->q_full);
           }
+          if (kind == 2 && s == 0) {
+            // the pass-2 item's queries (rows of its unit) into shared memory
+            if (!wait_bar(&ms->qs_empty, (qcount & 1) ^ 1, ms, p.status)) {
+              ok = false;
+              break;
+            }
+            const int layer = st.u2 / p.upl, local = st.u2 % p.upl;
+            const int b = local / p.Hkv, h = local % p.Hkv;
+            const int qrow0 = (b * p.Hq + h * p.G) * p.W;
+            mbar_arrive_expect_tx(&ms->qs_full, kTileBytes);
+            tma_load_2d(qsm, &lp.qmap[layer], 0, qrow0, &ms->qs_full);
+            tma_load_2d(qsm + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->qs_full);
+            ++qcount;
+          }
+          const int unit = pass == 1 ? st.u1 : st.u2;
+          const int tt = pass == 1 ? st.a0 + s : st.b0 + s;
+          const int ks = kcount % C::NK;
+          if (!wait_bar(&ms->k_empty[ks], ((kcount / C::NK) & 1) ^ 1, ms, p.status)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
+          uint8_t *kb = ktiles + ks * kTileBytes;
+          const uint64_t pol = pass == 1 ? keep : drop;
+          const CUtensorMap *km =
+              kind == 3 ? &lp.vmap[unit / p.upl] : &lp.kmap[unit / p.upl];
+          const int local = unit % p.upl;
+          tma_load_3d(kb, km, 0, tt * kTile, local, &ms->k_full[ks], pol);
+          tma_load_3d(kb + kHalfBytes, km, 64, tt * kTile, local, &ms->k_full[ks], pol);
+          ++kcount;
         }
       }
-      for (int j = max(0, kcount - kNK); j < kcount; ++j)
-        mbar_wait(&ms->k_full[j % kNK], (j / kNK) & 1, nullptr);
+      for (int j = max(0, kcount - C::NK); j < kcount; ++j)
+        mbar_wait(&ms->k_full[j % C::NK], (j / C::NK) & 1, nullptr);
       if (qcount > 0) mbar_wait(&ms->qs_full, (qcount - 1) & 1, nullptr);
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int kcount = 0, acount = 0, qcount = 0;
+      int kcount = 0, acount = 0, qcount = 0, pcount = 0, ocount = 0;
       constexpr uint32_t id = idesc_bf16(128, 128);
+      // O = P . V: P (rows x keys) and V (keys x dims) both MN-major
+      constexpr uint32_t id_pv = idesc_bf16(128, 128) | (1u << 15) | (1u << 16);
       const uint32_t kbase = smem_u32(ktiles), qsbase = smem_u32(qsm), q1base = smem_u32(q1m);
+      const uint32_t pbase = smem_u32(ptile);
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
         if (k < n && !wait_bar(&ms->q_full, k & 1, ms, p.status)) break;
-        for (int j = 0; j < st.len && ok; ++j) {
-          {
-            int pass, s;
+        const int len = kO ? st.n1 + 2 * st.n2 : st.len;
+        for (int j = 0; j < len && ok; ++j) {
+          int pass, s, kind;
+          if (kO) {
+            oseq_at(st, j, kind, s);
+            pass = kind == 1 ? 1 : 2;
+          } else {
             seq_at(st, j, pass, s);
-            if (pass == 2 && s == 0) {
-              if (st.n1 > 0) mma_commit(&ms->q_empty);  // item k's pass-1 queries are free
-              if (!wait_bar(&ms->qs_full, qcount & 1, ms, p.status)) {
-                ok = false;
-                break;
-              }
-            }
-            const int ks = kcount % kNK, as = acount % kNA;
-            if (!wait_bar(&ms->k_full[ks], (kcount / kNK) & 1, ms, p.status) ||
-                !wait_bar(&ms->acc_empty[as], ((acount / kNA) & 1) ^ 1, ms, p.status)) {
+            kind = pass;
+          }
+          const int ks = kcount % C::NK;
+          const uint32_t ka = kbase + ks * kTileBytes;
+          if (kO && kind == 3) {
+            // O (+)= P . V for pass-2 tile s, once the epilogue has written
+            // its probabilities (and, for the item's first tile, has read
+            // out the previous item's O)
+            if ((s == 0 && !wait_bar(&ms->o_empty, (ocount & 1) ^ 1, ms, p.status)) ||
+                !wait_bar(&ms->p_full, pcount & 1, ms, p.status) ||
+                !wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t d = tmem + as * 128;
-            const uint32_t ka = kbase + ks * kTileBytes;
-            if (pass == 1) {
 #pragma unroll
-              for (int kk = 0; kk < 8; ++kk) {
-                const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                mma_bf16(d, sw128_desc(q1base + off), sw128_desc(ka + off), id, kk > 0);
-              }
-            } else {
-#pragma unroll
-              for (int kk = 0; kk < 8; ++kk) {
-                const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                mma_bf16(d, sw128_desc(ka + off), sw128_desc(qsbase + off), id, kk > 0);
-              }
-            }
+            for (int kk = 0; kk < 8; ++kk)
+              mma_bf16(tmem + C::OCol, sw128_desc_mn(pbase + kk * 2048, kHalfBytes, 1024),
+                       sw128_desc_mn(ka + kk * 2048, kHalfBytes, 1024), id_pv, kk > 0 || s > 0);
             mma_commit(&ms->k_empty[ks]);
-            mma_commit(&ms->acc_full[as]);
+            mma_commit(&ms->p_empty);
             ++kcount;
-            ++acount;
+            ++pcount;
+            if (s == st.n2 - 1) {
+              mma_commit(&ms->o_full);
+              ++ocount;
+            }
+            continue;
           }
+          if (pass == 2 && s == 0) {
+            if (st.n1 > 0) mma_commit(&ms->q_empty);  // item k's pass-1 queries are free
+            if (!wait_bar(&ms->qs_full, qcount & 1, ms, p.status)) {
+              ok = false;
+              break;
+            }
+          }
+          const int as = acount % C::NA;
+          if (!wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status) ||
+              !wait_bar(&ms->acc_empty[as], ((acount / C::NA) & 1) ^ 1, ms, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d = tmem + as * 128;
+          if (pass == 1) {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+              mma_bf16(d, sw128_desc(q1base + off), sw128_desc(ka + off), id, kk > 0);
+            }
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+              mma_bf16(d, sw128_desc(ka + off), sw128_desc(qsbase + off), id, kk > 0);
+            }
+          }
+          mma_commit(&ms->k_empty[ks]);
+          mma_commit(&ms->acc_full[as]);
+          ++kcount;
+          ++acount;
         }
         if (ok && st.n2 > 0) {
           mma_commit(&ms->qs_empty);  // the pass-2 queries are free
@@ -424,6 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int wtid = threadIdx.x - 64 - wg * 128;
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     int tcount = 0;  // tiles seen
+    int pc = 0, oc = 0;  // kO: pass-2 tiles seen, pass-2 items seen
 
     // Inside an item every warp follows the same control flow even if a wait
     // gives up (the tile is then skipped), so that the named barriers below
@@ -439,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // ---------------- a pass-1 tile of item k
           const int t = st.a0 + s;
           const int mine = wg_of(tcount) == wg;
-          const int as = tcount % kNA, ph = (tcount / kNA) & 1;
+          const int as = tcount % C::NA, ph = (tcount / C::NA) & 1;
           ++tcount;
           if (mine && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
             tc_fence_after();
@@ -512,7 +649,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const int t = st.b0 + s;
           const int mine = wg_of(tcount) == wg;
-          const int as = tcount % kNA, ph = (tcount / kNA) & 1;
+          const int as = tcount % C::NA, ph = (tcount / C::NA) & 1;
           ++tcount;
           if (mine && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
             tc_fence_after();
@@ -529,6 +666,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
             const float2 s2 = make_float2(p.scale2, p.scale2);
             const float4 *o4 = reinterpret_cast<const float4 *>(ms->offs[wg]);
+            const int key = t * kTile + r;
+            // kO: a window key (or a key past the end) is seen only by the
+            // rows at or after it (causal inside the window)
+            const int hidden_below = kO && key >= p.P ? key - p.P : -1;
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
@@ -540,18 +681,101 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float2 y1 = __ffma2_rn(make_float2(__uint_as_float(x[c][4 * j4 + 2]),
                                                          __uint_as_float(x[c][4 * j4 + 3])),
                                              s2, make_float2(-o.z, -o.w));
-                sv[(2 * j4) & 3] =
-                    __fadd2_rn(sv[(2 * j4) & 3], make_float2(fast_exp2(y0.x), fast_exp2(y0.y)));
-                sv[(2 * j4 + 1) & 3] =
-                    __fadd2_rn(sv[(2 * j4 + 1) & 3], make_float2(fast_exp2(y1.x), fast_exp2(y1.y)));
+                float2 e0 = make_float2(fast_exp2(y0.x), fast_exp2(y0.y));
+                float2 e1 = make_float2(fast_exp2(y1.x), fast_exp2(y1.y));
+                if (kO) {
+                  if (hidden_below >= 0) {
+                    const int col = c * 32 + 4 * j4;  // window row of e0.x
+                    if ((col + 0) % p.W < hidden_below) e0.x = 0.f;
+                    if ((col + 1) % p.W < hidden_below) e0.y = 0.f;
+                    if ((col + 2) % p.W < hidden_below) e1.x = 0.f;
+                    if ((col + 3) % p.W < hidden_below) e1.y = 0.f;
+                  }
+                  x[c][4 * j4] = __float_as_uint(e0.x);
+                  x[c][4 * j4 + 1] = __float_as_uint(e0.y);
+                  x[c][4 * j4 + 2] = __float_as_uint(e1.x);
+                  x[c][4 * j4 + 3] = __float_as_uint(e1.y);
+                }
+                sv[(2 * j4) & 3] = __fadd2_rn(sv[(2 * j4) & 3], e0);
+                sv[(2 * j4 + 1) & 3] = __fadd2_rn(sv[(2 * j4 + 1) & 3], e1);
               }
             const float vote = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
                                ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
-            const int key = t * kTile + r;
+            if (kO) {
+              // this key's probabilities of the 128 rows into the tile the
+              // MMA warp multiplies by the value tile, once it has read the
+              // previous tile's
+              warp_wait(&ms->p_empty, (pc & 1) ^ 1, ms, p.status);
+              store_p_row(ptile, r, x);
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&ms->p_full);
+            }
             if (key < p.P)
               p.votes[guard((long long)st.u2 * p.P + key, 1, (long long)p.units * p.P, p.status)] =
                   vote;
           }
+          if (kO) ++pc;
+        }
+      }
+      if (kO && st.n2 > 0) {
+        // ---------------- kO: item k - kLag's partial O (both warpgroups:
+        // this thread's row, warpgroup wg's 64 dims), and the unit's output
+        // from its items' partials, summed in item order by the item that
+        // completes the unit
+        const ItemRef it = item_of(p, k - kLag);
+        const size_t prow = ((size_t)it.unit * p.n_ch + it.chunk) * 128 + r;
+        if (warp_wait(&ms->o_full, oc & 1, ms, p.status)) {
+          tc_fence_after();
+          uint32_t x[2][32];
+          tmem_ld32(tmem + lane_addr + C::OCol + wg * 64, x[0]);
+          tmem_ld32(tmem + lane_addr + C::OCol + wg * 64 + 32, x[1]);
+          tmem_wait_ld();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ms->o_empty);
+          float4 *dst = reinterpret_cast<float4 *>(
+              p.o_part + guard((long long)prow * 128 + wg * 64, 64,
+                               (long long)p.units * p.n_ch * 128 * 128, p.status));
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            dst[i] = make_float4(__uint_as_float(x[i >> 3][(i & 7) * 4]),
+                                 __uint_as_float(x[i >> 3][(i & 7) * 4 + 1]),
+                                 __uint_as_float(x[i >> 3][(i & 7) * 4 + 2]),
+                                 __uint_as_float(x[i >> 3][(i & 7) * 4 + 3]));
+        }
+        ++oc;
+        __threadfence();
+        named_bar_sync(5, 256);
+        if (wg == 0 && wtid == 0)
+          ms->o_last = atomicAdd(&p.o_count[guard(it.unit, 1, p.units, p.status)], 1) == p.n_ch - 1;
+        named_bar_sync(5, 256);
+        if (ms->o_last) {
+          __threadfence();
+          float4 acc[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+          const size_t ubase = (size_t)it.unit * p.n_ch * 128;
+          for (int c = 0; c < p.n_ch; ++c) {
+            const float4 *src = reinterpret_cast<const float4 *>(
+                p.o_part + ((ubase + (size_t)c * 128 + r) * 128 + wg * 64));
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float4 v4 = __ldcg(src + i);
+              acc[i].x += v4.x;
+              acc[i].y += v4.y;
+              acc[i].z += v4.z;
+              acc[i].w += v4.w;
+            }
+          }
+          const int layer = it.unit / p.upl, local = it.unit % p.upl;
+          const int b = local / p.Hkv, h = local % p.Hkv;
+          const long long orow = (long long)(b * p.Hq + h * p.G) * p.W + r;
+          float4 *out = reinterpret_cast<float4 *>(
+              p.o_win[layer] + guard(orow * 128 + wg * 64, 64,
+                                     (long long)p.upl / p.Hkv * p.Hq * p.W * 128, p.status));
+#pragma unroll
+          for (int i = 0; i < 16; ++i) out[i] = acc[i];
         }
       }
     }
@@ -565,6 +789,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_dealloc(tmem, 512);
   }
 }
+
 
 // ------------------------------------------------------------ host side
 
@@ -588,15 +813,24 @@ EncodeTiledFn encode_fn() {
 
 }  // namespace
 
+int score_tc1_max_items(const LayerGeom &g) {
+  const int n_tiles = (g.T + kTile - 1) / kTile;
+  return (n_tiles + kMinTilesPerItem - 1) / kMinTilesPerItem;
+}
+
 bool score_tc1_supported(const LayerGeom &g) {
   return g.dtype == RIPPLE_BF16 && g.D == 128 && g.R == 128 && g.P > 0 && encode_fn() != nullptr;
 }
 
 cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const *q_win,
                              const void *const *k, const CompressWs &ws, float *votes,
-                             int32_t *status, cudaStream_t st) {
+                             int32_t *status, cudaStream_t st, const void *const *v,
+                             float *const *o_win) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr || n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorNotSupported;
+  const bool with_o = v != nullptr;
+  if (with_o && (o_win == nullptr || ws.o_part == nullptr || ws.o_count == nullptr))
+    return cudaErrorInvalidValue;
   static Tc1Launch lp;  // large: kept off the stack, filled under the lock
   static std::mutex mu;
   std::lock_guard<std::mutex> lock(mu);
@@ -606,6 +840,11 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
     cuuint32_t box[3] = {64, 128, 1};
     cuuint32_t es[3] = {1, 1, 1};
     if (enc(&lp.kmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k[l]), dims,
+            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+    if (with_o &&
+        enc(&lp.vmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(v[l]), dims,
             strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
@@ -632,7 +871,7 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
   p.Hkv = g.Hkv;
   p.G = g.G;
   p.n_tiles1 = (g.T + kTile - 1) / kTile;
-  p.n_tiles2 = (g.P + kTile - 1) / kTile;
+  p.n_tiles2 = with_o ? p.n_tiles1 : (g.P + kTile - 1) / kTile;
   // At least kMinTilesPerItem tiles per item, and no more items per unit than
   // SMs (the deadlock-free schedule needs <= 2x as many as CTAs).
   const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
@@ -640,7 +879,9 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
   p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
   p.total_items = p.units * p.n_ch;
   p.scale2 = g.scale2;
-  for (int l = 0; l < n_layers; ++l) p.q[l] = (const uint8_t *)q_win[l];
+  for (int l = 0; l < n_layers; ++l) p.o_win[l] = with_o ? o_win[l] : nullptr;
+  p.o_part = with_o ? ws.o_part : nullptr;
+  p.o_count = with_o ? ws.o_count : nullptr;
   p.partial = ws.row_partial;
   p.lognorm = ws.row_lognorm;
   p.votes = votes;
@@ -648,14 +889,16 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
   p.status = status;
   p.wait_cycles = wait_limit_cycles();
   cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * p.units, st);
+  if (e == cudaSuccess && with_o) e = cudaMemsetAsync(ws.o_count, 0, sizeof(int) * p.units, st);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(score_tc1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           kSmemBytes);
+  const void *kernel = with_o ? (const void *)score_tc1_kernel<true>
+                              : (const void *)score_tc1_kernel<false>;
+  const int smem = with_o ? Tc1Smem<true>::Bytes : Tc1Smem<false>::Bytes;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const int grid = p.total_items < sms ? p.total_items : sms;
   void *args[] = {(void *)&lp};
-  e = cudaLaunchCooperativeKernel((const void *)score_tc1_kernel, dim3(grid), dim3(kThreads), args,
-                                  (size_t)kSmemBytes, st);
+  e = cudaLaunchCooperativeKernel(kernel, dim3(grid), dim3(kThreads), args, (size_t)smem, st);
   count_launches(1);
   return e;
 }

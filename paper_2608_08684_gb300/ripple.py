@@ -80,6 +80,17 @@ _lib.ripple_compress_layers.argtypes = [ctypes.POINTER(LayerDesc), _i32, ctypes.
                                         ctypes.POINTER(_i32), ctypes.POINTER(_p),
                                         ctypes.POINTER(_i32), _p, _sz, _p, _p]
 _lib.ripple_compress_layers.restype = _i32
+_lib.ripple_compress_layers_attn_workspace_bytes.argtypes = [ctypes.POINTER(LayerDesc), _i32,
+                                                             ctypes.POINTER(_sz)]
+_lib.ripple_compress_layers_attn_workspace_bytes.restype = _i32
+_lib.ripple_compress_layers_attn.argtypes = [ctypes.POINTER(LayerDesc), _i32,
+                                             ctypes.POINTER(_i64), ctypes.POINTER(_p),
+                                             ctypes.POINTER(_p), ctypes.POINTER(_p),
+                                             ctypes.POINTER(_p), ctypes.POINTER(_p),
+                                             ctypes.POINTER(_i32), ctypes.POINTER(_p),
+                                             ctypes.POINTER(_i32), ctypes.POINTER(_p), _p, _sz,
+                                             _p, _p]
+_lib.ripple_compress_layers_attn.restype = _i32
 _lib.ripple_select_layer.argtypes = [ctypes.POINTER(LayerDesc), _i64, _p, _p, _p, _p, _p, _i32, _p,
                                      ctypes.POINTER(_i32), _p, _sz, _p, _p]
 _lib.ripple_select_layer.restype = _i32
@@ -226,6 +237,33 @@ def ripple_compress_layers(desc: LayerDesc, budgets, tables: CompressTables, wor
                                        workspace.numel() * workspace.element_size(),
                                        _ptr(dev_status), _stream(stream)),
            "ripple_compress_layers")
+    return [int(x) for x in n]
+
+
+def ripple_compress_layers_attn_workspace_bytes(desc: LayerDesc, n_layers: int) -> int:
+    out = _sz()
+    _check(_lib.ripple_compress_layers_attn_workspace_bytes(ctypes.byref(desc), int(n_layers),
+                                                            ctypes.byref(out)),
+           "ripple_compress_layers_attn_workspace_bytes")
+    return out.value
+
+
+def ripple_compress_layers_attn(desc: LayerDesc, budgets, tables: CompressTables, o_win,
+                                workspace, dev_status=None, stream=None) -> list:
+    """ripple_compress_layers that also writes each layer's window-row attention
+    output into o_win[l] (fp32 [B][Hq][w][d]); returns n_l per layer."""
+    L = tables.n_layers
+    if len(o_win) != L:
+        raise ValueError("one o_win tensor per layer")
+    b = (_i64 * L)(*[int(x) for x in budgets])
+    n = (_i32 * L)()
+    o = (_p * L)(*[_ptr(x) for x in o_win])
+    _check(_lib.ripple_compress_layers_attn(ctypes.byref(desc), L, b, tables.q, tables.k,
+                                            tables.v, tables.k_out, tables.v_out, tables.caps,
+                                            tables.idx, n, o, _ptr(workspace),
+                                            workspace.numel() * workspace.element_size(),
+                                            _ptr(dev_status), _stream(stream)),
+           "ripple_compress_layers_attn")
     return [int(x) for x in n]
 
 

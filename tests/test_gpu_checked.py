@@ -165,3 +165,33 @@ def test_window_kl_checked(lib, chk, n_sets, n_pos, vocab, dtype):
         runs.append((int(status.item()), d_out, kl_out))
     assert runs[1][0] == 0
     assert torch.equal(runs[0][1], runs[1][1]) and torch.equal(runs[0][2], runs[1][2])
+
+
+def test_compress_layers_attn_checked(lib, chk):
+    # the scoring fused into the window rows' prefill attention (several items
+    # per unit, window keys across the last tiles)
+    wl = synth.WORKLOADS["tiny"].replace(n_layers=2, batch=1, n_q_heads=8, n_kv_heads=2,
+                                         head_dim=128, seq_len=2100, dtype="bf16", seed=68)
+    budgets = [300, 1500]
+    B, H, d = wl.batch, wl.n_kv_heads, wl.head_dim
+    ins = [tuple(t.to(DEV) for t in C.layer_inputs(wl, l, "cpu")) for l in range(wl.n_layers)]
+    results = []
+    for m in (lib, chk):
+        desc = m.layer_desc(B, wl.n_q_heads, H, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                            wl.torch_dtype)
+        ns = [m.ripple_keep_count(x, wl.seq_len, wl.window) for x in budgets]
+        k_out = [torch.zeros(B, H, n, d, dtype=wl.torch_dtype, device=DEV) for n in ns]
+        v_out = [torch.zeros_like(x) for x in k_out]
+        idx = [torch.full((B * H * n,), -1, dtype=torch.int32, device=DEV) for n in ns]
+        o_win = [torch.empty(B, wl.n_q_heads, wl.window, d, device=DEV) for _ in ns]
+        tables = m.CompressTables([x[0] for x in ins], [x[1] for x in ins], [x[2] for x in ins],
+                                  k_out, v_out, idx)
+        ws = torch.empty(m.ripple_compress_layers_attn_workspace_bytes(desc, wl.n_layers),
+                         dtype=torch.uint8, device=DEV)
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        m.ripple_compress_layers_attn(desc, budgets, tables, o_win, ws, dev_status=status)
+        torch.cuda.synchronize()
+        results.append((int(status.item()), idx + k_out + v_out + o_win))
+    assert results[1][0] == 0
+    for x, y in zip(results[0][1], results[1][1]):
+        assert torch.equal(x, y)

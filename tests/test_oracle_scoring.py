@@ -232,3 +232,51 @@ def test_decode_closed_forms():
     v9 = _rand((9, 32), 5)
     np.testing.assert_allclose(O.decode_attention(q, k, v9, 0.2), np.tile(v9.mean(0), (4, 1)),
                                rtol=1e-12, atol=1e-14)
+
+
+# ------------------------------------------- window rows' prefill attention
+
+
+@pytest.mark.parametrize("G,w,T,d", [(1, 1, 1, 4), (2, 4, 12, 3), (4, 32, 300, 16), (8, 7, 7, 5)])
+def test_window_attention_matches_torch_sdpa(G, w, T, d):
+    # the window rows of a causal prefill attention: torch's scaled dot-product
+    # attention over all T queries with its own causal mask, last w rows taken
+    rng = np.random.default_rng(7 + G + T)
+    q_all = rng.standard_normal((G, T, d))
+    k = 2.0 * rng.standard_normal((T, d))
+    v = rng.standard_normal((T, d))
+    scale = 1.0 / math.sqrt(d)
+    got = O.window_attention(q_all[:, T - w:], k, v, scale)
+    t = lambda a: torch.from_numpy(a)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        t(q_all)[None], t(k)[None, None].expand(1, G, T, d), t(v)[None, None].expand(1, G, T, d),
+        is_causal=True, scale=scale)[0, :, T - w:].numpy()
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-13)
+
+
+def test_window_attention_closed_forms():
+    G, w, T, d = 2, 5, 9, 4
+    P = T - w
+    rng = np.random.default_rng(11)
+    q = rng.standard_normal((G, w, d))
+    v = rng.standard_normal((T, d))
+    # identical keys: row i averages the P + i + 1 values it can see
+    k = np.tile(rng.standard_normal(d), (T, 1))
+    got = O.window_attention(q, k, v, 0.5)
+    for i in range(w):
+        np.testing.assert_allclose(got[:, i], np.tile(v[:P + i + 1].mean(0), (G, 1)), rtol=1e-12)
+    # one token: the value itself
+    one = O.window_attention(q[:, :1], k[:1], v[:1], 0.5)
+    np.testing.assert_allclose(one, np.tile(v[0], (G, 1, 1)), rtol=0, atol=0)
+    # the row's probabilities are those the votes add up: with one-hot value
+    # columns the output is the row's attention over the keys, and its sum
+    # over rows is the vote of every key
+    kk = rng.standard_normal((T, d))
+    votes, _, _ = O.window_votes(q, kk, 0.5)
+    probs = O.window_attention(q, kk, np.eye(T), 0.5)
+    assert probs.shape == (G, w, T)
+    np.testing.assert_allclose(probs.sum(axis=2), 1.0, rtol=1e-12)
+    np.testing.assert_allclose(probs.sum(axis=(0, 1)), votes, rtol=1e-12)
+    # the causal mask: a row never weights a later window token
+    for i in range(w):
+        assert np.all(probs[:, i, P + i + 1:] == 0)
