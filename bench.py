@@ -61,7 +61,7 @@ def parse_args():
                     help="skip the other workloads and the serving-loop measurement")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target CPU seconds of the oracle sample")
-    ap.add_argument("--case", choices=["compress", "decode", "perturb", "kl", "serve"],
+    ap.add_argument("--case", choices=["compress", "attn", "decode", "perturb", "kl", "serve"],
                     default=None,
                     help="time one entry point alone (one layer / one decode step / the "
                          "profiling kernels: Eq. 6 perturbation of one layer's V cache, Eq. 7 "
@@ -100,6 +100,8 @@ def run_case(args):
     times = []
     if args.case in ("perturb", "kl"):
         return run_profile_case(args, R, synth, wl, dev)
+    if args.case == "attn":
+        return run_attn_case(args, R, synth, wl, dev, budgets, n_keep)
     if args.case == "serve":
         line = {"case": "serve", "workload": wl.name}
         line.update(serving_loop_measure(R, synth, wl, dev, min(args.repeat * 4, wl.decode_steps)))
@@ -188,6 +190,73 @@ def run_case(args):
                       "ms_per_call": round(ms, 5), "bytes_per_call": nbytes,
                       "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
                       "peak_source": src}), flush=True)
+
+
+def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
+    """The scoring fused into the prefill attention of the window rows
+    (ripple_compress_layers_attn) on the args.layers largest-budget layers in
+    one call (every layer reading the same K/V, inputs above L2), beside
+    ripple_compress_layers on the same inputs. Algorithmic bytes of the fused
+    call: the compression's, plus V read in full and the fp32 outputs. The
+    separate alternative would read the window rows' K and V once more (the
+    prefill attention of those rows): `separate_read_ms` is that read at the
+    measured copy bandwidth."""
+    import torch
+    L, B, Hq, Hkv, d, e = (wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim,
+                           wl.elem_bytes)
+    nl = max(1, args.layers)
+    lay = sorted(range(L), key=lambda i: -budgets[i])[:nl]
+    layer = lay[0]
+    q_win = synth.layer_window_queries(wl, layer, dev)
+    k = synth.layer_keys(wl, layer, dev)
+    v = synth.layer_values(wl, layer, dev)
+    desc = R.layer_desc(B, Hq, Hkv, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                        wl.torch_dtype)
+    outs = [(torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
+             torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
+             torch.empty(B * Hkv * n_keep[i], dtype=torch.int32, device=dev)) for i in lay]
+    tabs = R.CompressTables([q_win] * nl, [k] * nl, [v] * nl, [o[0] for o in outs],
+                            [o[1] for o in outs], [o[2] for o in outs])
+    o_win = [torch.empty(B, Hq, wl.window, d, device=dev) for _ in lay]
+    ws_a = torch.empty(R.ripple_compress_layers_attn_workspace_bytes(desc, nl), dtype=torch.uint8,
+                       device=dev)
+    ws_c = torch.empty(R.ripple_compress_layers_workspace_bytes(desc, nl), dtype=torch.uint8,
+                       device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    bud = [budgets[i] for i in lay]
+    comp_bytes = sum(B * Hkv * d * e * (wl.seq_len + 3 * n_keep[i]) + B * Hq * wl.window * d * e
+                     for i in lay)
+    attn_bytes = comp_bytes + nl * (B * Hkv * wl.seq_len * d * e + B * Hq * wl.window * d * 4)
+
+    def timed(fn):
+        ts = []
+        for i in range(args.repeat + 2):
+            a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b_.record()
+            if i >= 2:
+                ts.append((a, b_))
+        torch.cuda.synchronize()
+        return statistics.mean(a.elapsed_time(b) for a, b in ts)
+
+    ms_a = timed(lambda: R.ripple_compress_layers_attn(desc, bud, tabs, o_win, ws_a,
+                                                       dev_status=status))
+    ms_c = timed(lambda: R.ripple_compress_layers(desc, bud, tabs, ws_c, dev_status=status))
+    assert int(status.item()) == 0, int(status.item())
+    hbm, src = measured_peaks()
+    kv_bytes = nl * 2 * B * Hkv * wl.seq_len * d * e
+    gbs = attn_bytes / (ms_a / 1e3) / 1e9
+    print(json.dumps({
+        "case": "attn", "workload": wl.name,
+        "what": (f"compress {nl} layers with the window rows' attention output in one call "
+                 f"(budgets of layers {lay}, K/V of layer {layer})"),
+        "calls": args.repeat, "ms_per_call": round(ms_a, 5), "bytes_per_call": attn_bytes,
+        "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
+        "compress_only_ms": round(ms_c, 5),
+        "extra_ms_for_outputs": round(ms_a - ms_c, 5),
+        "separate_read_ms": round(kv_bytes / (hbm * 1e9) * 1e3, 5),
+        "peak_source": src}), flush=True)
 
 
 def run_profile_case(args, R, synth, wl, dev):

@@ -31,8 +31,12 @@
 // accumulates O[row][dim] += P . V in the last 128 TMEM columns (V, MN-major,
 // the B operand). The probabilities are final (pass 1 has fixed every row's
 // normaliser), so O needs no rescaling. At an item's end both warpgroups
-// write its partial O to the workspace; the item that completes its unit
-// sums the unit's partials in item order into the output.
+// write its partial O to the workspace and count it on its unit. kOReduceLag
+// steps later the CTA that computed the item sums its slice of the unit's
+// output rows (a 1/n_ch share) over the unit's partials in item order (the
+// unit's other items are done by then; a bounded wait covers the rest), so
+// the sum is deterministic and no CTA holds up the others with a whole
+// unit's sum.
 #include <cuda.h>
 #include <math.h>
 
@@ -53,6 +57,7 @@ constexpr int kLag = 1;                         // pass 2 of item k runs in step
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
 constexpr int kMaxStages = 4;
+constexpr int kOReduceLag = 2;  // kO: a step's item rows are summed this many steps later
 
 // With kO (the window rows' attention output as well as the votes) pass 2
 // covers every key and also streams the value tiles, multiplies the
@@ -154,10 +159,12 @@ struct Misc {
   uint64_t acc_full[kMaxStages], acc_empty[kMaxStages];
   uint64_t qs_full, qs_empty;           // pass-2 queries in shared memory
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
-  uint64_t p_full, p_empty, o_full, o_empty;  // kO: probability tile, O accumulator
+  // kO: the probability tile, per writing warpgroup (the tiles alternate
+  // between the warpgroups, but not strictly across a step's pass-1 tiles, and
+  // a parity wait only tells apart phases one apart), and the O accumulator
+  uint64_t p_full[2], p_empty[2], o_full, o_empty;
   uint32_t tmem_base;
   int abort_flag;
-  int o_last;                           // kO: this CTA completed its unit's partials
   long long wait_cycles;  // bound of the waits of this launch
   float2 pstat[kPubSlots][2][128];      // pass-1 row statistics per slot and warpgroup
   alignas(16) float offs[2][128];       // per warpgroup: the pass-2 item's row log-normalisers
@@ -229,10 +236,13 @@ struct Tc1Launch {
 };
 
 // With kO the producer and the MMA warp walk a step as: the pass-1 key tiles,
-// then for the pass-2 item key tile s followed by value tile s - 1 (the order
-// the MMA warp consumes them in: it multiplies a tile's probabilities by its
-// values after issuing the next tile's logits), then the last value tile.
+// then the pass-2 item's key tiles with value tile s - kPvLag after key tile
+// s (the order the MMA warp consumes them in: it multiplies a tile's
+// probabilities by its values after issuing the logits kPvLag tiles on, so
+// that the warpgroup that has just written a tile's probabilities finds its
+// next tile's logits done), then the last value tiles.
 // kind 1: pass-1 key tile, 2: pass-2 key tile, 3: pass-2 value tile.
+constexpr int kPvLag = 2;
 __device__ __forceinline__ void oseq_at(const Step &s, int j, int &kind, int &idx) {
   if (j < s.n1) {
     kind = 1;
@@ -240,43 +250,86 @@ __device__ __forceinline__ void oseq_at(const Step &s, int j, int &kind, int &id
     return;
   }
   const int q = j - s.n1;
-  if (q == 0) {
+  const int a = min(s.n2, kPvLag);           // leading key tiles
+  const int pairs = max(0, s.n2 - kPvLag);   // (key s, value s - kPvLag)
+  if (q < a) {
     kind = 2;
-    idx = 0;
-  } else if (q == 2 * s.n2 - 1) {
-    kind = 3;
-    idx = s.n2 - 1;
-  } else if (q & 1) {
-    kind = 2;
-    idx = (q + 1) >> 1;
+    idx = q;
+  } else if (q - a < 2 * pairs) {
+    const int t = (q - a) >> 1;
+    kind = (q - a) & 1 ? 3 : 2;
+    idx = (q - a) & 1 ? t : kPvLag + t;
   } else {
     kind = 3;
-    idx = (q >> 1) - 1;
+    idx = pairs + (q - a - 2 * pairs);
   }
 }
 
-// Probabilities of one key (this thread's TMEM lane) for the 128 window rows
-// (fp32 bit patterns, row e in pr[e / 32][e % 32]), as bf16, into the shared-memory tile in the MN-major, 128-byte-swizzled
-// layout the tensor core reads as the A operand of O = P . V: rows 0-63 and
-// 64-127 in two 16 KB halves, in each the key's 128-byte line holds its 64
-// rows, 16-byte chunk c at position c ^ (key mod 8).
-__device__ __forceinline__ void store_p_row(uint8_t *ptile, int key, const uint32_t (&pr)[4][32]) {
+// Probabilities of one key (this thread's TMEM lane) for the 128 window rows,
+// as bf16 pairs (rows 2i and 2i + 1 in pk[i]), into the shared-memory tile in
+// the MN-major, 128-byte-swizzled layout the tensor core reads as the A
+// operand of O = P . V: rows 0-63 and 64-127 in two 16 KB halves, in each the
+// key's 128-byte line holds its 64 rows, 16-byte chunk c at position
+// c ^ (key mod 8).
+__device__ __forceinline__ void store_p_row(uint8_t *ptile, int key, const uint32_t (&pk)[64]) {
 #pragma unroll
   for (int half = 0; half < 2; ++half)
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-      uint32_t w[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const int e = half * 64 + c * 8 + 2 * i;  // rows e, e + 1
-        const __nv_bfloat162 b = __floats2bfloat162_rn(__uint_as_float(pr[e >> 5][e & 31]),
-                                                       __uint_as_float(pr[(e + 1) >> 5][(e + 1) & 31]));
-        w[i] = *reinterpret_cast<const uint32_t *>(&b);
-      }
+      const int w = half * 32 + c * 4;  // rows 8c .. 8c + 7 of the half
       uint8_t *dst = ptile + half * kHalfBytes + (key >> 3) * 1024 + (key & 7) * 128 +
                      ((c ^ (key & 7)) << 4);
-      *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+      *reinterpret_cast<uint4 *>(dst) = make_uint4(pk[w], pk[w + 1], pk[w + 2], pk[w + 3]);
     }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t *>(&b);
+}
+
+// kO: the output rows of item `it`'s slice of its unit (rows chunk * 128 /
+// n_ch up to the next chunk's), summed over the unit's item partials in item
+// order, once every item of the unit has written its partial (bounded wait).
+// Run by both epilogue warpgroups (256 threads, named barrier 5).
+__device__ __forceinline__ void reduce_rows(const Tc1Params &p, Misc *ms, const ItemRef &it,
+                                            int tid) {
+  if (tid == 0) {
+    const int *cnt = &p.o_count[guard(it.unit, 1, p.units, p.status)];
+    const long long t0 = clock64();
+    while (ld_acquire(cnt) < p.n_ch) {
+      if (*(volatile int *)&ms->abort_flag) break;
+      if (clock64() - t0 > ms->wait_cycles) {
+        *(volatile int *)&ms->abort_flag = 1;
+        report(p.status, RIPPLE_ETIMEOUT);
+        break;
+      }
+      __nanosleep(64);
+    }
+  }
+  named_bar_sync(5, 256);
+  const int r0 = it.chunk * 128 / p.n_ch, r1 = (it.chunk + 1) * 128 / p.n_ch;
+  const int layer = it.unit / p.upl, local = it.unit % p.upl;
+  const int b = local / p.Hkv, h = local % p.Hkv;
+  const long long orow0 = (long long)(b * p.Hq + h * p.G) * p.W;
+  const size_t ubase = (size_t)it.unit * p.n_ch * 128;
+  // 32 float4 per row; consecutive threads take consecutive float4
+  for (int e = tid; e < (r1 - r0) * 32; e += 256) {
+    const int row = r0 + (e >> 5), q4 = e & 31;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = 0; c < p.n_ch; ++c) {
+      const float4 v4 = __ldcg(reinterpret_cast<const float4 *>(
+                                   p.o_part + (ubase + (size_t)c * 128 + row) * 128) +
+                               q4);
+      acc.x += v4.x;
+      acc.y += v4.y;
+      acc.z += v4.z;
+      acc.w += v4.w;
+    }
+    reinterpret_cast<float4 *>(
+        p.o_win[layer] + guard((orow0 + row) * 128, 128,
+                               (long long)p.upl / p.Hkv * p.Hq * p.W * 128, p.status))[q4] = acc;
+  }
 }
 
 template <bool kO>
@@ -313,12 +366,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->pub_empty[i], 1);
     }
     mbar_init(&ms->mma_done, 1);
-    mbar_init(&ms->p_full, 4);
-    mbar_init(&ms->p_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ms->p_full[i], 4);
+      mbar_init(&ms->p_empty[i], 1);
+    }
     mbar_init(&ms->o_full, 1);
     mbar_init(&ms->o_empty, 8);
     ms->abort_flag = 0;
-    ms->o_last = 0;
     ms->wait_cycles = p.wait_cycles;
     fence_mbar_init();
   }
@@ -341,6 +395,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
         const int len = kO ? st.n1 + 2 * st.n2 : st.len;
+        if (kO && st.n2 > 0) {
+          // the pass-2 item's value tiles into L2 while the step's pass-1
+          // tiles stream from DRAM (the ring has little room to run ahead)
+          const CUtensorMap *vm = &lp.vmap[st.u2 / p.upl];
+          const int local = st.u2 % p.upl;
+          for (int s2 = 0; s2 < st.n2; ++s2) {
+            tma_prefetch_3d(vm, 0, (st.b0 + s2) * kTile, local);
+            tma_prefetch_3d(vm, 64, (st.b0 + s2) * kTile, local);
+          }
+        }
         for (int j = 0; j < len && ok; ++j) {
           int pass, s, kind;
           if (kO) {
@@ -403,7 +467,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
-      int kcount = 0, acount = 0, qcount = 0, pcount = 0, ocount = 0;
+      int kcount = 0, acount = 0, qcount = 0, ocount = 0;
+      // kO: bit s mod 4 = the warpgroup that writes pass-2 tile s's
+      // probabilities; tiles consumed per writing warpgroup
+      uint32_t pv_owner = 0;
+      int pv_count0 = 0, pv_count1 = 0;
       constexpr uint32_t id = idesc_bf16(128, 128);
       // O = P . V: P (rows x keys) and V (keys x dims) both MN-major
       constexpr uint32_t id_pv = idesc_bf16(128, 128) | (1u << 15) | (1u << 16);
@@ -429,8 +497,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             // O (+)= P . V for pass-2 tile s, once the epilogue has written
             // its probabilities (and, for the item's first tile, has read
             // out the previous item's O)
+            static_assert(kPvLag + 2 <= 32, "owner bits");
+            const int ow = (pv_owner >> (s % (kPvLag + 2))) & 1;
+            const int pvc = ow ? pv_count1 : pv_count0;
             if ((s == 0 && !wait_bar(&ms->o_empty, (ocount & 1) ^ 1, ms, p.status)) ||
-                !wait_bar(&ms->p_full, pcount & 1, ms, p.status) ||
+                !wait_bar(&ms->p_full[ow], pvc & 1, ms, p.status) ||
                 !wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status)) {
               ok = false;
               break;
@@ -441,9 +512,12 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(tmem + C::OCol, sw128_desc_mn(pbase + kk * 2048, kHalfBytes, 1024),
                        sw128_desc_mn(ka + kk * 2048, kHalfBytes, 1024), id_pv, kk > 0 || s > 0);
             mma_commit(&ms->k_empty[ks]);
-            mma_commit(&ms->p_empty);
+            mma_commit(&ms->p_empty[ow]);
             ++kcount;
-            ++pcount;
+            if (ow)
+              ++pv_count1;
+            else
+              ++pv_count0;
             if (s == st.n2 - 1) {
               mma_commit(&ms->o_full);
               ++ocount;
@@ -458,6 +532,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           const int as = acount % C::NA;
+          if (kO && kind == 2) {
+            const uint32_t bit = 1u << (s % (kPvLag + 2));
+            pv_owner = wg_of(acount) ? pv_owner | bit : pv_owner & ~bit;
+          }
           if (!wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status) ||
               !wait_bar(&ms->acc_empty[as], ((acount / C::NA) & 1) ^ 1, ms, p.status)) {
             ok = false;
@@ -560,7 +638,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int wtid = threadIdx.x - 64 - wg * 128;
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     int tcount = 0;  // tiles seen
-    int pc = 0, oc = 0;  // kO: pass-2 tiles seen, pass-2 items seen
+    int oc = 0;            // kO: pass-2 items seen
+    int pw0 = 0, pw1 = 0;  // kO: probability tiles written, per warpgroup
+    int prev_writer = -1;  // kO: the warpgroup that wrote the previous tile
 
     // Inside an item every warp follows the same control flow even if a wait
     // gives up (the tile is then skipped), so that the named barriers below
@@ -670,6 +750,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // kO: a window key (or a key past the end) is seen only by the
             // rows at or after it (causal inside the window)
             const int hidden_below = kO && key >= p.P ? key - p.P : -1;
+            uint32_t pk[kO ? 64 : 1];  // kO: the probabilities as bf16 pairs
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
@@ -683,7 +764,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                              s2, make_float2(-o.z, -o.w));
                 float2 e0 = make_float2(fast_exp2(y0.x), fast_exp2(y0.y));
                 float2 e1 = make_float2(fast_exp2(y1.x), fast_exp2(y1.y));
-                if (kO) {
+                if constexpr (kO) {
                   if (hidden_below >= 0) {
                     const int col = c * 32 + 4 * j4;  // window row of e0.x
                     if ((col + 0) % p.W < hidden_below) e0.x = 0.f;
@@ -691,31 +772,40 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if ((col + 2) % p.W < hidden_below) e1.x = 0.f;
                     if ((col + 3) % p.W < hidden_below) e1.y = 0.f;
                   }
-                  x[c][4 * j4] = __float_as_uint(e0.x);
-                  x[c][4 * j4 + 1] = __float_as_uint(e0.y);
-                  x[c][4 * j4 + 2] = __float_as_uint(e1.x);
-                  x[c][4 * j4 + 3] = __float_as_uint(e1.y);
+                  pk[(c * 32 + 4 * j4) >> 1] = pack_bf16x2(e0.x, e0.y);
+                  pk[((c * 32 + 4 * j4) >> 1) + 1] = pack_bf16x2(e1.x, e1.y);
                 }
                 sv[(2 * j4) & 3] = __fadd2_rn(sv[(2 * j4) & 3], e0);
                 sv[(2 * j4 + 1) & 3] = __fadd2_rn(sv[(2 * j4 + 1) & 3], e1);
               }
             const float vote = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
                                ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
-            if (kO) {
+            if constexpr (kO) {
               // this key's probabilities of the 128 rows into the tile the
               // MMA warp multiplies by the value tile, once it has read the
               // previous tile's
-              warp_wait(&ms->p_empty, (pc & 1) ^ 1, ms, p.status);
-              store_p_row(ptile, r, x);
+              // once the previous tile's probabilities have been multiplied
+              // (its writer's pw[.] - 1-th phase)
+              if (prev_writer >= 0)
+                warp_wait(&ms->p_empty[prev_writer], ((prev_writer ? pw1 : pw0) - 1) & 1, ms,
+                          p.status);
+              store_p_row(ptile, r, pk);
               fence_proxy_async_smem();
               __syncwarp();
-              if (lane == 0) mbar_arrive(&ms->p_full);
+              if (lane == 0) mbar_arrive(&ms->p_full[wg]);
             }
             if (key < p.P)
               p.votes[guard((long long)st.u2 * p.P + key, 1, (long long)p.units * p.P, p.status)] =
                   vote;
           }
-          if (kO) ++pc;
+          if (kO) {
+            const int writer = wg_of(tcount - 1);
+            if (writer)
+              ++pw1;
+            else
+              ++pw0;
+            prev_writer = writer;
+          }
         }
       }
       if (kO && st.n2 > 0) {
@@ -745,40 +835,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                                  __uint_as_float(x[i >> 3][(i & 7) * 4 + 3]));
         }
         ++oc;
+        // count the item once every row of its partial is written
         __threadfence();
         named_bar_sync(5, 256);
-        if (wg == 0 && wtid == 0)
-          ms->o_last = atomicAdd(&p.o_count[guard(it.unit, 1, p.units, p.status)], 1) == p.n_ch - 1;
-        named_bar_sync(5, 256);
-        if (ms->o_last) {
-          __threadfence();
-          float4 acc[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-          const size_t ubase = (size_t)it.unit * p.n_ch * 128;
-          for (int c = 0; c < p.n_ch; ++c) {
-            const float4 *src = reinterpret_cast<const float4 *>(
-                p.o_part + ((ubase + (size_t)c * 128 + r) * 128 + wg * 64));
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float4 v4 = __ldcg(src + i);
-              acc[i].x += v4.x;
-              acc[i].y += v4.y;
-              acc[i].z += v4.z;
-              acc[i].w += v4.w;
-            }
-          }
-          const int layer = it.unit / p.upl, local = it.unit % p.upl;
-          const int b = local / p.Hkv, h = local % p.Hkv;
-          const long long orow = (long long)(b * p.Hq + h * p.G) * p.W + r;
-          float4 *out = reinterpret_cast<float4 *>(
-              p.o_win[layer] + guard(orow * 128 + wg * 64, 64,
-                                     (long long)p.upl / p.Hkv * p.Hq * p.W * 128, p.status));
-#pragma unroll
-          for (int i = 0; i < 16; ++i) out[i] = acc[i];
-        }
+        if (wg == 0 && wtid == 0) atomicAdd(&p.o_count[guard(it.unit, 1, p.units, p.status)], 1);
       }
+      // kO: this CTA's slice of the output rows of the unit of its pass-2
+      // item of kOReduceLag steps ago (its other items are done by then)
+      if (kO && k - kOReduceLag >= kLag) reduce_rows(p, ms, item_of(p, k - kOReduceLag - kLag), wg * 128 + wtid);
     }
+    // kO: the slices whose steps would come after the last one
+    if (kO)
+      for (int kr = max(kLag, n + kLag - kOReduceLag); kr < n + kLag; ++kr)
+        reduce_rows(p, ms, item_of(p, kr - kLag), wg * 128 + wtid);
   }
 
   tc_fence_before();
