@@ -56,6 +56,7 @@ constexpr int kThreads = 352;
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
+constexpr int kMinTilesPerItemO = 9;  // kO: the same, with the values and partials in L2 too
 constexpr int kMaxStages = 4;
 constexpr int kOReduceLag = 2;  // kO: a step's item rows are summed this many steps later
 
@@ -395,16 +396,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
         const int len = kO ? st.n1 + 2 * st.n2 : st.len;
-        if (kO && st.n2 > 0) {
-          // the pass-2 item's value tiles into L2 while the step's pass-1
-          // tiles stream from DRAM (the ring has little room to run ahead)
-          const CUtensorMap *vm = &lp.vmap[st.u2 / p.upl];
-          const int local = st.u2 % p.upl;
-          for (int s2 = 0; s2 < st.n2; ++s2) {
-            tma_prefetch_3d(vm, 0, (st.b0 + s2) * kTile, local);
-            tma_prefetch_3d(vm, 64, (st.b0 + s2) * kTile, local);
-          }
-        }
         for (int j = 0; j < len && ok; ++j) {
           int pass, s, kind;
           if (kO) {
@@ -884,7 +875,7 @@ EncodeTiledFn encode_fn() {
 
 int score_tc1_max_items(const LayerGeom &g) {
   const int n_tiles = (g.T + kTile - 1) / kTile;
-  return (n_tiles + kMinTilesPerItem - 1) / kMinTilesPerItem;
+  return (n_tiles + kMinTilesPerItemO - 1) / kMinTilesPerItemO;
 }
 
 bool score_tc1_supported(const LayerGeom &g) {
@@ -944,7 +935,8 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
   // At least kMinTilesPerItem tiles per item, and no more items per unit than
   // SMs (the deadlock-free schedule needs <= 2x as many as CTAs).
   const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
-  p.tpi = tpi_min > kMinTilesPerItem ? tpi_min : kMinTilesPerItem;
+  const int tpi_floor = with_o ? kMinTilesPerItemO : kMinTilesPerItem;
+  p.tpi = tpi_min > tpi_floor ? tpi_min : tpi_floor;
   p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
   p.total_items = p.units * p.n_ch;
   p.scale2 = g.scale2;
