@@ -193,8 +193,14 @@ def run_case(args):
 
 
 def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
+    print(json.dumps(dict({"case": "attn", "workload": wl.name},
+                          **attn_measure(R, synth, wl, dev, budgets, n_keep, args.layers,
+                                         args.repeat))), flush=True)
+
+
+def attn_measure(R, synth, wl, dev, budgets, n_keep, n_layers, repeat):
     """The scoring fused into the prefill attention of the window rows
-    (ripple_compress_layers_attn) on the args.layers largest-budget layers in
+    (ripple_compress_layers_attn) on the n_layers largest-budget layers in
     one call (every layer reading the same K/V, inputs above L2), beside
     ripple_compress_layers on the same inputs. Algorithmic bytes of the fused
     call: the compression's, plus V read in full and the fp32 outputs. The
@@ -204,7 +210,7 @@ def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
     import torch
     L, B, Hq, Hkv, d, e = (wl.n_layers, wl.batch, wl.n_q_heads, wl.n_kv_heads, wl.head_dim,
                            wl.elem_bytes)
-    nl = max(1, args.layers)
+    nl = max(1, min(n_layers, L))
     lay = sorted(range(L), key=lambda i: -budgets[i])[:nl]
     layer = lay[0]
     q_win = synth.layer_window_queries(wl, layer, dev)
@@ -230,7 +236,7 @@ def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
 
     def timed(fn):
         ts = []
-        for i in range(args.repeat + 2):
+        for i in range(repeat + 2):
             a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record()
             fn()
@@ -247,16 +253,15 @@ def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
     hbm, src = measured_peaks()
     kv_bytes = nl * 2 * B * Hkv * wl.seq_len * d * e
     gbs = attn_bytes / (ms_a / 1e3) / 1e9
-    print(json.dumps({
-        "case": "attn", "workload": wl.name,
+    return {
         "what": (f"compress {nl} layers with the window rows' attention output in one call "
                  f"(budgets of layers {lay}, K/V of layer {layer})"),
-        "calls": args.repeat, "ms_per_call": round(ms_a, 5), "bytes_per_call": attn_bytes,
+        "calls": repeat, "ms_per_call": round(ms_a, 5), "bytes_per_call": attn_bytes,
         "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
         "compress_only_ms": round(ms_c, 5),
         "extra_ms_for_outputs": round(ms_a - ms_c, 5),
         "separate_read_ms": round(kv_bytes / (hbm * 1e9) * 1e3, 5),
-        "peak_source": src}), flush=True)
+        "peak_source": src}
 
 
 def run_profile_case(args, R, synth, wl, dev):
@@ -781,7 +786,7 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(st, args.cpu_seconds)
     budgets = st.budgets
-    others = serving = None
+    others = serving = fused = None
     if rank == 0 and world == 1 and not args.no_workloads:
         # the other workloads and the per-layer serving loop, after the
         # headline workload's buffers are freed
@@ -791,6 +796,10 @@ def run_ours(args, rank, world, local_rank):
             others = measure_workloads(R, synth, device,
                                        [n for n in synth.WORKLOADS if n != args.workload], 3)
             serving = serving_loop_measure(R, synth, wl, device, 32)
+            fused = attn_measure(R, synth, wl, device, budgets,
+                                 [R.ripple_keep_count(b, wl.seq_len, wl.window) for b in budgets],
+                                 wl.n_layers, 3) if wl.dtype == "bf16" and wl.head_dim == 128 \
+                and wl.group * wl.window == 128 else None
         others["clocks"] = oclocks.summary()
     if rank != 0:
         return
@@ -818,6 +827,8 @@ def run_ours(args, rank, world, local_rank):
     if others:
         line["workloads"] = others
         line["serving_loop"] = serving
+        if fused:
+            line["compress_attn"] = fused
     if cpu:
         line["cpu_baseline"] = cpu
     print(json.dumps(line), flush=True)
