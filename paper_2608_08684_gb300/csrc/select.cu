@@ -500,31 +500,36 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
 
 // Prefixes up to kUMaxP tokens: one 1024-thread CTA per unit and no cluster
 // (a launch covers every unit of every layer, so the GPU is filled by units).
-// The pooled keys stay in registers, key j = i * 1024 + thread (i < 32), so
-// that staging, pooling and every radix round read shared memory with
-// consecutive lanes on consecutive words; four radix rounds of 8 bits count
-// into per-warp histograms (no contention between warps); the ordered
-// compaction takes each warp's ballots per row of 1024 keys and one block
-// scan over the (row, warp) counts. Same result as select_kernel, bit for bit.
+// Thread t keeps the pooled keys of tokens 32t .. 32t + 31 in registers: the
+// votes are staged in shared memory with a pad word after every 32 (coalesced
+// stores, conflict-free reads of a thread's run), the 7-wide max pooling is
+// three maxima per key over the run and its halo, four radix rounds of 8 bits
+// count into per-warp histograms (no contention between warps), and the
+// ordered compaction is one block scan over the threads' counts followed by
+// each thread writing its kept tokens in order. Same result as select_kernel,
+// bit for bit.
 constexpr int kUThreads = 1024;
 constexpr int kUWarps = kUThreads / 32;
 constexpr int kUKeys = 32;                    // keys per thread
 constexpr int kUMaxP = kUThreads * kUKeys;
 constexpr int kUBins = 256;
 constexpr int kUMinUnits = 256;               // units per launch for this kernel
+constexpr int kUCand = 128;                   // bucket size that ends the radix rounds
 // shared words before the staged votes: per-warp histograms, bin totals,
-// (row, warp) counts, scan scratch and control
-constexpr int kUHead = kUWarps * kUBins + kUBins + kUKeys * kUWarps + 64;
+// scan scratch and control
+constexpr int kUHead = kUWarps * kUBins + kUBins + 64;
+
+// Shared-memory word of staged vote j: one pad word after every 32.
+__device__ __forceinline__ int upad(int j) { return j + (j >> 5); }
 
 __global__ void __launch_bounds__(kUThreads, 1)
     select_unit_kernel(LayerGeom g, const float *votes, const __grid_constant__ SelTable tab) {
   extern __shared__ uint32_t sm[];
   uint32_t *hist = sm;                                   // [kUWarps][kUBins]
   int *tot = (int *)(hist + kUWarps * kUBins);           // [kUBins]
-  int *cnt = tot + kUBins;                               // [kUKeys][kUWarps], packed (gt << 16) | eq
-  int *warp_tot = cnt + kUKeys * kUWarps;                // [33]
-  int *ctl = warp_tot + 40;                              // [2]
-  float *vs = reinterpret_cast<float *>(sm + kUHead);    // [P]
+  int *warp_tot = tot + kUBins;                          // [33]
+  int *ctl = warp_tot + 40;                              // [6]
+  float *vs = reinterpret_cast<float *>(sm + kUHead);    // [P + P / 32], padded
 
   const int unit = blockIdx.x;  // over all layers of the launch
   const int layer = unit / tab.upl;
@@ -541,62 +546,85 @@ __global__ void __launch_bounds__(kUThreads, 1)
     return;
   }
 
-  // Votes into shared memory, eight loads of a thread in flight at once.
+  // Votes into shared memory (coalesced, sixteen loads of a thread in flight),
+  // with one pad word after every 32: thread t then reads its run of keys
+  // 32t .. 32t + 31 (and the pooling halo) without bank conflicts.
 #pragma unroll
-  for (int i0 = 0; i0 < kUKeys; i0 += 8) {
-    float x[8];
+  for (int i0 = 0; i0 < kUKeys; i0 += 16) {
+    float x[16];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       const int j = (i0 + u) * kUThreads + tid;
       x[u] = j < P ? __ldcg(v + j) : 0.f;
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       const int j = (i0 + u) * kUThreads + tid;
-      if (j < P) vs[j] = x[u];
+      if (j < P) vs[upad(j)] = x[u];
     }
   }
   __syncthreads();
 
-  // Pooled keys (window clipped to the prefix).
+  // Pooled keys of this thread's tokens j0 .. j0 + 31 (window clipped to the
+  // prefix).
   const int half = g.pool_kernel / 2;
+  const int j0 = tid * kUKeys;
   uint32_t key[kUKeys];
+  if (g.pool_type == RIPPLE_POOL_MAX && half == 3) {
+    // the 7-wide max from the votes w = v[j0 - 3 .. j0 + 34] (-inf outside
+    // the prefix): b[i] = max(w[i .. i + 3]) and pooled(j0 + i) = max(b[i], b[i + 3])
+    float w[kUKeys + 6];
 #pragma unroll
-  for (int i = 0; i < kUKeys; ++i) {
-    const int j = i * kUThreads + tid;
-    float r = 0.f;
-    if (j < P) {
-      if (g.pool_type == RIPPLE_POOL_MAX && half == 3 && j >= 3 && j + 3 < P) {
-        // the 7-wide window away from the prefix edges (almost every key)
-        r = fmaxf(fmaxf(fmaxf(vs[j - 3], vs[j - 2]), fmaxf(vs[j - 1], vs[j])),
-                  fmaxf(fmaxf(vs[j + 1], vs[j + 2]), vs[j + 3]));
-      } else if (g.pool_type == RIPPLE_POOL_MAX) {
-        r = vs[j];
-        for (int d = 1; d <= half; ++d) {
-          if (j - d >= 0) r = fmaxf(r, vs[j - d]);
-          if (j + d < P) r = fmaxf(r, vs[j + d]);
-        }
-      } else if (g.pool_type == RIPPLE_POOL_AVG) {
-        float sum = 0.f;
-        int c = 0;
-        for (int d = -half; d <= half; ++d) {
-          const int pos = j + d;
-          if (pos >= 0 && pos < P) {
-            sum = __fadd_rn(sum, vs[pos]);
-            ++c;
-          }
-        }
-        r = __fdiv_rn(sum, (float)c);
-      } else {
-        r = vs[j];
-      }
+    for (int i = 0; i < kUKeys + 6; ++i) {
+      const int j = j0 - 3 + i;
+      w[i] = j >= 0 && j < P ? vs[upad(j)] : -INFINITY;
     }
-    key[i] = order_key(r);
+    float a[kUKeys + 5];
+#pragma unroll
+    for (int i = 0; i < kUKeys + 5; ++i) a[i] = fmaxf(w[i], w[i + 1]);
+    float b[kUKeys + 3];
+#pragma unroll
+    for (int i = 0; i < kUKeys + 3; ++i) b[i] = fmaxf(a[i], a[i + 2]);
+#pragma unroll
+    for (int i = 0; i < kUKeys; ++i) key[i] = order_key(fmaxf(b[i], b[i + 3]));
+  } else {
+#pragma unroll
+    for (int i = 0; i < kUKeys; ++i) {
+      const int j = j0 + i;
+      float r = 0.f;
+      if (j < P) {
+        if (g.pool_type == RIPPLE_POOL_MAX) {
+          r = vs[upad(j)];
+          for (int d = 1; d <= half; ++d) {
+            if (j - d >= 0) r = fmaxf(r, vs[upad(j - d)]);
+            if (j + d < P) r = fmaxf(r, vs[upad(j + d)]);
+          }
+        } else if (g.pool_type == RIPPLE_POOL_AVG) {
+          float sum = 0.f;
+          int c = 0;
+          for (int d = -half; d <= half; ++d) {
+            const int pos = j + d;
+            if (pos >= 0 && pos < P) {
+              sum = __fadd_rn(sum, vs[upad(pos)]);
+              ++c;
+            }
+          }
+          r = __fdiv_rn(sum, (float)c);
+        } else {
+          r = vs[upad(j)];
+        }
+      }
+      key[i] = order_key(r);
+    }
   }
 
-  // Radix select of the K-th largest key: 4 rounds of 8 bits from the top.
+  // Radix select of the K-th largest key: up to 4 rounds of 8 bits from the
+  // top; once the bucket that holds it has at most kUCand keys, the rest is
+  // found among that bucket's keys directly (tau is then the same key).
   uint32_t prefix = 0, mask = 0;
   int remaining = K;
+  uint32_t tau = 0;
+  int take_eq = -1;
   uint32_t *hw = hist + wid * kUBins;
   for (int round = 0; round < 4; ++round) {
     const int shift = 24 - 8 * round;
@@ -604,10 +632,8 @@ __global__ void __launch_bounds__(kUThreads, 1)
     for (int b = lane; b < kUBins; b += 32) hw[b] = 0;
     __syncwarp();
 #pragma unroll
-    for (int i = 0; i < kUKeys; ++i) {
-      const int j = i * kUThreads + tid;
-      if (j < P && (key[i] & mask) == prefix) atomicAdd(&hw[(key[i] >> shift) & 255u], 1u);
-    }
+    for (int i = 0; i < kUKeys; ++i)
+      if (j0 + i < P && (key[i] & mask) == prefix) atomicAdd(&hw[(key[i] >> shift) & 255u], 1u);
     __syncthreads();
     if (tid < kUBins) {
       int sum = 0;
@@ -636,46 +662,69 @@ __global__ void __launch_bounds__(kUThreads, 1)
         if (above < remaining && remaining <= above + c[q]) {
           ctl[0] = kUBins - 1 - 8 * lane - q;
           ctl[1] = remaining - above;
+          ctl[2] = c[q];
         }
         above += c[q];
       }
+      if (lane == 0) ctl[3] = 0;
     }
     __syncthreads();
     prefix |= (uint32_t)ctl[0] << shift;
     mask |= 255u << shift;
     remaining = ctl[1];
+    if (round < 3 && ctl[2] <= kUCand) {
+      // the bucket's keys into a list (any order); each of them counts the
+      // keys above and equal to it, and the one with remaining - 1 above
+      // and at least remaining above or equal is tau
+      uint32_t *cand = hist;  // the histograms are not needed any more
+#pragma unroll
+      for (int i = 0; i < kUKeys; ++i)
+        if (j0 + i < P && (key[i] & mask) == prefix) cand[atomicAdd(&ctl[3], 1)] = key[i];
+      __syncthreads();
+      const int nc = ctl[2];
+      if (tid < nc) {
+        const uint32_t x = cand[tid];
+        int above = 0, same = 0;
+        for (int c = 0; c < nc; ++c) {
+          const uint32_t y = cand[c];
+          above += y > x;
+          same += y == x;
+        }
+        if (above < remaining && remaining <= above + same) {
+          ctl[4] = (int)x;
+          ctl[5] = remaining - above;
+        }
+      }
+      __syncthreads();
+      tau = (uint32_t)ctl[4];
+      take_eq = ctl[5];
+      break;
+    }
   }
-  const uint32_t tau = prefix;
-  const int take_eq = remaining;
+  if (take_eq < 0) {
+    tau = prefix;
+    take_eq = remaining;
+  }
 
-  // Ordered compaction: per row i of 1024 keys and warp w, the counts of keys
-  // above tau and equal to tau; one block scan over (row, warp) in key order.
+  // Ordered compaction: this thread's counts of keys above and equal to tau,
+  // one block scan over the threads (token order), then its kept tokens in
+  // order: every key above tau and the first take_eq keys equal to it.
+  int gt = 0, eq = 0;
 #pragma unroll
   for (int i = 0; i < kUKeys; ++i) {
-    const int j = i * kUThreads + tid;
-    const int gt = __popc(__ballot_sync(0xffffffffu, j < P && key[i] > tau));
-    const int eq = __popc(__ballot_sync(0xffffffffu, j < P && key[i] == tau));
-    if (lane == 0) cnt[i * kUWarps + wid] = (gt << 16) | eq;
+    gt += j0 + i < P && key[i] > tau;
+    eq += j0 + i < P && key[i] == tau;
   }
-  __syncthreads();
-  {
-    int total;
-    const int x = cnt[tid];  // entry (row tid / 32, warp tid % 32)
-    const int off = block_exclusive_scan(x, warp_tot, &total);
-    cnt[tid] = off;
-  }
-  __syncthreads();
-  const uint32_t below = (1u << lane) - 1u;
+  int total;
+  const int off = block_exclusive_scan((gt << 16) | eq, warp_tot, &total);
+  int g_rank = off >> 16, e_rank = off & 0xffff;
 #pragma unroll
   for (int i = 0; i < kUKeys; ++i) {
-    const int j = i * kUThreads + tid;
-    const bool gt = j < P && key[i] > tau, eq = j < P && key[i] == tau;
-    const uint32_t bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
-    const int off = cnt[i * kUWarps + wid];
-    const int g_rank = (off >> 16) + __popc(bg & below);
-    const int e_rank = (off & 0xffff) + __popc(be & below);
-    if (gt || (eq && e_rank < take_eq))
-      out[guard(g_rank + min(e_rank, take_eq), 1, K, tab.status)] = j;
+    const bool is_gt = j0 + i < P && key[i] > tau, is_eq = j0 + i < P && key[i] == tau;
+    if (is_gt || (is_eq && e_rank < take_eq))
+      out[guard(g_rank + min(e_rank, take_eq), 1, K, tab.status)] = j0 + i;
+    g_rank += is_gt;
+    e_rank += is_eq;
   }
 }
 
@@ -695,7 +744,7 @@ cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
       tab.n_keep[l] = n_keep[l];
       tab.idx[l] = idx[l];
     }
-    const size_t smem = sizeof(uint32_t) * ((size_t)kUHead + g.P);
+    const size_t smem = sizeof(uint32_t) * ((size_t)kUHead + g.P + g.P / 32 + 1);
     cudaError_t e = cudaFuncSetAttribute(select_unit_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
