@@ -240,14 +240,19 @@ static ripple_status compress_layers_impl(
                                    : carve_layers_ws(g, n_layers, workspace);
   if (workspace_bytes < ws.bytes) return RIPPLE_EWORKSPACE;
   cudaStream_t st = (cudaStream_t)stream;
+  // selection and gather in one launch where the selection kernel takes both
+  const GatherArgs ga{k_host, v_host, k_out_host, v_out_host, cap};
+  bool gathered = false;
   if (g.P > 0 && score_tc1_supported(g)) {
-    // All layers in three launches: scoring, selection, gather.
+    // All layers in two or three launches: scoring, selection (+ gather).
     RIPPLE_CUDA_TRY(launch_score_tc1(g, n_layers, q_win_host, k_host, ws, ws.votes, dev_status,
                                      st, o_win_host ? v_host : nullptr, o_win_host));
-    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st));
-    RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
-                                  (const int32_t *const *)idx_out_host, n, k_out_host,
-                                  v_out_host, cap, dev_status, st));
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st,
+                                  &ga, &gathered));
+    if (!gathered)
+      RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
+                                    (const int32_t *const *)idx_out_host, n, k_out_host,
+                                    v_out_host, cap, dev_status, st));
   } else {
     // Other shapes: scoring layer by layer (each layer's votes in its part of
     // the vote array, the scratch of the multi-layer workspace reused), then
@@ -262,10 +267,12 @@ static ripple_status compress_layers_impl(
                                               dev_status, st);
       RIPPLE_CUDA_TRY(e);
     }
-    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st));
-    RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
-                                  (const int32_t *const *)idx_out_host, n, k_out_host,
-                                  v_out_host, cap, dev_status, st));
+    RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st,
+                                  &ga, &gathered));
+    if (!gathered)
+      RIPPLE_CUDA_TRY(launch_gather(g, n_layers, k_host, v_host,
+                                    (const int32_t *const *)idx_out_host, n, k_out_host,
+                                    v_out_host, cap, dev_status, st));
   }
   for (int l = 0; l < n_layers; ++l) n_keep_host[l] = n[l];
   return RIPPLE_OK;

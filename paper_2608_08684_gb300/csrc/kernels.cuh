@@ -66,11 +66,22 @@ cudaError_t launch_score_tc1(const LayerGeom &g, int n_layers, const void *const
                              float *const *o_win = nullptr);
 // Items per unit of launch_score_tc1 at most (sizes the output partials).
 int score_tc1_max_items(const LayerGeom &g);
+// The gather's inputs and outputs per layer (launch_gather's arguments).
+struct GatherArgs {
+  const void *const *k;
+  const void *const *v;
+  void *const *k_out;
+  void *const *v_out;
+  const int *cap;
+};
 // Pooling + exact top-k per unit of n_layers layers (votes [n_layers][units][P]);
-// writes idx[l] [units][n_keep[l]].
+// writes idx[l] [units][n_keep[l]]. With gather and gathered given, the
+// kernel may also gather the kept rows (as launch_gather would); *gathered
+// says whether it did.
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
                           const CompressWs &ws, const int *n_keep, int32_t *const *idx,
-                          int32_t *status, cudaStream_t st);
+                          int32_t *status, cudaStream_t st, const GatherArgs *gather = nullptr,
+                          bool *gathered = nullptr);
 // idx = 0..T-1 for every unit (keep-all case).
 cudaError_t launch_iota(const LayerGeom &g, int32_t *idx, cudaStream_t st);
 // Gather kept K and V rows of n_layers layers into [units][cap[l]][d].

@@ -294,6 +294,13 @@ struct SelTable {
   int n_keep[kCompressMaxLayers];
   int32_t *idx[kCompressMaxLayers];
   int32_t *status;
+  // select_unit_kernel with gather != 0 also copies each unit's kept rows
+  int gather, row_bytes;
+  const uint8_t *k[kCompressMaxLayers];
+  const uint8_t *v[kCompressMaxLayers];
+  uint8_t *k_out[kCompressMaxLayers];
+  uint8_t *v_out[kCompressMaxLayers];
+  int cap[kCompressMaxLayers];
 };
 
 __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
@@ -522,29 +529,17 @@ constexpr int kUHead = kUWarps * kUBins + kUBins + 64;
 // Shared-memory word of staged vote j: one pad word after every 32.
 __device__ __forceinline__ int upad(int j) { return j + (j >> 5); }
 
-__global__ void __launch_bounds__(kUThreads, 1)
-    select_unit_kernel(LayerGeom g, const float *votes, const __grid_constant__ SelTable tab) {
-  extern __shared__ uint32_t sm[];
+// Pooling, radix select and ordered compaction of one unit's prefix tokens
+// (0 < K < P): writes out[0 .. K).
+__device__ __forceinline__ void select_unit_keys(const LayerGeom &g, const float *v, int32_t *out,
+                                                 int K, uint32_t *sm, int32_t *status) {
   uint32_t *hist = sm;                                   // [kUWarps][kUBins]
   int *tot = (int *)(hist + kUWarps * kUBins);           // [kUBins]
   int *warp_tot = tot + kUBins;                          // [33]
   int *ctl = warp_tot + 40;                              // [6]
   float *vs = reinterpret_cast<float *>(sm + kUHead);    // [P + P / 32], padded
-
-  const int unit = blockIdx.x;  // over all layers of the launch
-  const int layer = unit / tab.upl;
-  const int n_keep = tab.n_keep[layer];
-  const int P = g.P, K = n_keep - g.W;
-  const float *v = votes + (size_t)unit * P;
-  int32_t *out = tab.idx[layer] + (size_t)(unit % tab.upl) * n_keep;
+  const int P = g.P;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
-
-  for (int j = tid; j < g.W; j += kUThreads) out[K + j] = P + j;
-  if (K <= 0) return;
-  if (K >= P) {
-    for (int t = tid; t < P; t += kUThreads) out[t] = t;
-    return;
-  }
 
   // Votes into shared memory (coalesced, sixteen loads of a thread in flight),
   // with one pad word after every 32: thread t then reads its run of keys
@@ -722,9 +717,60 @@ __global__ void __launch_bounds__(kUThreads, 1)
   for (int i = 0; i < kUKeys; ++i) {
     const bool is_gt = j0 + i < P && key[i] > tau, is_eq = j0 + i < P && key[i] == tau;
     if (is_gt || (is_eq && e_rank < take_eq))
-      out[guard(g_rank + min(e_rank, take_eq), 1, K, tab.status)] = j0 + i;
+      out[guard(g_rank + min(e_rank, take_eq), 1, K, status)] = j0 + i;
     g_rank += is_gt;
     e_rank += is_eq;
+  }
+}
+
+__global__ void __launch_bounds__(kUThreads, 1)
+    select_unit_kernel(LayerGeom g, const float *votes, const __grid_constant__ SelTable tab) {
+  extern __shared__ uint32_t sm[];
+  const int unit = blockIdx.x;  // over all layers of the launch
+  const int layer = unit / tab.upl;
+  const int n_keep = tab.n_keep[layer];
+  const int P = g.P, K = n_keep - g.W;
+  int32_t *out = tab.idx[layer] + (size_t)(unit % tab.upl) * n_keep;
+  const int tid = threadIdx.x;
+
+  for (int j = tid; j < g.W; j += kUThreads) out[K + j] = P + j;
+  if (K >= P) {
+    for (int t = tid; t < P; t += kUThreads) out[t] = t;
+  } else if (K > 0) {
+    select_unit_keys(g, votes + (size_t)unit * P, out, K, sm, tab.status);
+  }
+  if (tab.gather) {
+    // the unit's kept K and V rows into its compact cache rows 0 .. n_keep - 1:
+    // row_bytes / 16 consecutive threads copy one row 16 bytes each, four rows
+    // a thread in flight
+    __syncthreads();  // out[] of this CTA written
+    const int rb = tab.row_bytes, lpr = rb >> 4, rpp = kUThreads / lpr;
+    const int r_in = tid / lpr, c16 = (tid % lpr) * 16;
+    const size_t local = (size_t)(unit % tab.upl);
+    const uint8_t *kin = tab.k[layer] + local * g.T * rb;
+    const uint8_t *vin = tab.v[layer] + local * g.T * rb;
+    uint8_t *kout = tab.k_out[layer] + local * tab.cap[layer] * rb;
+    uint8_t *vout = tab.v_out[layer] + local * tab.cap[layer] * rb;
+    for (int r0 = 0; r0 < n_keep; r0 += 4 * rpp) {
+      uint4 xk[4], xv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int r = r0 + u * rpp + r_in;
+        if (r < n_keep) {
+          const long long t = guard(__ldcg(&out[r]), 1, g.T, tab.status);
+          xk[u] = __ldcs(reinterpret_cast<const uint4 *>(kin + t * rb + c16));
+          xv[u] = __ldcs(reinterpret_cast<const uint4 *>(vin + t * rb + c16));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int r = r0 + u * rpp + r_in;
+        if (r < n_keep) {
+          *reinterpret_cast<uint4 *>(kout + (size_t)r * rb + c16) = xk[u];
+          *reinterpret_cast<uint4 *>(vout + (size_t)r * rb + c16) = xv[u];
+        }
+      }
+    }
   }
 }
 
@@ -732,17 +778,28 @@ __global__ void __launch_bounds__(kUThreads, 1)
 
 cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
                           const CompressWs &ws, const int *n_keep, int32_t *const *idx,
-                          int32_t *status, cudaStream_t st) {
+                          int32_t *status, cudaStream_t st, const GatherArgs *gather,
+                          bool *gathered) {
   if (n_layers < 1 || n_layers > kCompressMaxLayers) return cudaErrorInvalidValue;
+  if (gathered != nullptr) *gathered = false;
   // One CTA per unit once the launch has enough units to fill the GPU;
   // fewer units (a single layer) are spread over 8-CTA clusters instead.
   if (g.P <= kUMaxP && (long long)g.units * n_layers >= kUMinUnits) {
     SelTable tab;
     tab.upl = g.units;
     tab.status = status;
+    tab.gather = gather != nullptr && gathered != nullptr;
+    tab.row_bytes = g.D * (g.dtype == RIPPLE_F32 ? 4 : 2);
     for (int l = 0; l < n_layers; ++l) {
       tab.n_keep[l] = n_keep[l];
       tab.idx[l] = idx[l];
+      if (tab.gather) {
+        tab.k[l] = (const uint8_t *)gather->k[l];
+        tab.v[l] = (const uint8_t *)gather->v[l];
+        tab.k_out[l] = (uint8_t *)gather->k_out[l];
+        tab.v_out[l] = (uint8_t *)gather->v_out[l];
+        tab.cap[l] = gather->cap[l];
+      }
     }
     const size_t smem = sizeof(uint32_t) * ((size_t)kUHead + g.P + g.P / 32 + 1);
     cudaError_t e = cudaFuncSetAttribute(select_unit_kernel,
@@ -750,13 +807,16 @@ cudaError_t launch_select(const LayerGeom &g, int n_layers, const float *votes,
     if (e != cudaSuccess) return e;
     select_unit_kernel<<<g.units * n_layers, kUThreads, smem, st>>>(g, votes, tab);
     count_launches(1);
-    return cudaGetLastError();
+    e = cudaGetLastError();
+    if (e == cudaSuccess && gathered != nullptr) *gathered = tab.gather != 0;
+    return e;
   }
   const int per_cta = ((g.P + kCluster - 1) / kCluster + 31) & ~31;
   if (per_cta <= kCMaxKeys && (long long)g.units * n_layers * kCluster <= 0x7fffffff) {
     SelTable tab;
     tab.upl = g.units;
     tab.status = status;
+    tab.gather = 0;
     for (int l = 0; l < n_layers; ++l) {
       tab.n_keep[l] = n_keep[l];
       tab.idx[l] = idx[l];
