@@ -773,8 +773,8 @@ def run_ours(args, rank, world, local_rank):
                                     "llama3-8b_B4_T32768_8layers.md), scaled to all layers by "
                                     "algorithmic bytes")
                  if comp_traffic else None,
-                 "kernel": ("score_tc1_kernel + select_unit_kernel + gather_kernel "
-                            "(ripple_compress_layers, all layers in three launches)"),
+                 "kernel": ("score_tc1_kernel + select_unit_kernel (with the gather) "
+                            "(ripple_compress_layers, all layers in two launches)"),
                  "bytes_per_launch": round(st.compress_bytes()),
                  "ms_per_launch": round(comp_avg, 4), "peak_source": hbm_src}
     dominant = roof_dec if dec_total >= comp_total else roof_comp

@@ -181,8 +181,9 @@ ripple_status ripple_compress_layers_workspace_bytes(const ripple_layer_desc *de
  * same shape (same desc) in one call, each with its own budget (the budgets
  * b_l of Eqs. 9-12). Layer l's result is exactly that of ripple_compress_layer
  * with budgets_host[l] and layer l's buffers; the layers are processed
- * together (bf16, d = 128, G * w = 128: three launches for all layers, so the
- * GPU is not idle between layers), otherwise one after another.
+ * together (bf16, d = 128, G * w = 128: two launches for all layers, scoring
+ * and selection with the gather, so the GPU is not idle between layers),
+ * otherwise one after another.
  *
  * n_layers     1..RIPPLE_COMPRESS_MAX_LAYERS, and n_layers * B * Hkv <= 65535
  * budgets_host host [n_layers]
