@@ -522,12 +522,14 @@ class Serving:
         self.ctables = R.CompressTables(self.q_win, self.k, self.v, self.k_out, self.v_out,
                                         self.idx)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
-        self.dq, self.dk, self.dv = [], [], []
-        for t in range(wl.decode_steps):
-            q, kn, vn = synth.decode_inputs(wl, t, device)
-            self.dq.append(q)
-            self.dk.append(kn)
-            self.dv.append(vn)
+        # every decode step's inputs in one tensor per kind (dq[t] is a view),
+        # so that the end-to-end run copies them in three copies
+        steps = [synth.decode_inputs(wl, t, device) for t in range(wl.decode_steps)]
+        self.dq_all, self.dk_all, self.dv_all = (torch.stack([x[i] for x in steps])
+                                                 for i in range(3))
+        del steps
+        self.dq, self.dk, self.dv = (list(x.unbind(0))
+                                     for x in (self.dq_all, self.dk_all, self.dv_all))
         self.ddesc = R.decode_desc(L, B, Hq, Hkv, d, wl.torch_dtype)
         self.tables = R.DecodeTables(self.k_out, self.v_out)
         self.dws = torch.empty(R.ripple_decode_workspace_bytes(self.ddesc, self.caps),
@@ -763,12 +765,12 @@ def run_ours(args, rank, world, local_rank):
                 "bytes_per_launch": round(st.decode_bytes_per_step()),
                 "ms_per_launch": round(dec_avg, 5), "peak_source": hbm_src}
     comp_traffic = profile_traffic("compress_kernels_llama3-8b_B4_T32768_8layers.md",
-                                   ["score_tc1.cu", "select.cu", "gather.cu", "tc_ptx.cuh",
-                                    "common.cuh"], st.compress_bytes()) \
+                                   ["score_tc1.cu", "select.cu", "tc_ptx.cuh", "common.cuh"],
+                                   st.compress_bytes()) \
         if wl.name.startswith("llama3-8b-32L-32q8kv-d128-B4-T32768") else None
     roof_comp = {"bound": "hbm", "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s",
                  "frac": round(comp_gbs / hbm, 4), "traffic": comp_traffic,
-                 "traffic_source": ("ncu dram bytes of the three kernels on an 8-layer "
+                 "traffic_source": ("ncu dram bytes of the two kernels on an 8-layer "
                                     "ripple_compress_layers call (profiles/compress_kernels_"
                                     "llama3-8b_B4_T32768_8layers.md), scaled to all layers by "
                                     "algorithmic bytes")
@@ -834,11 +836,17 @@ def run_ours(args, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
-def measure_e2e(st, args, torch, tokens):
+def measure_e2e(st, args, torch, tokens, group=8):
     """Same metric through the C ABI from pinned host buffers: every step copies
     the layer inputs and decode inputs host->device and reads the decode
-    outputs back, inside the timed region."""
-    wl = st.wl
+    outputs back, inside the timed region. The copies run on a second stream
+    in groups of `group` layers; each group is compressed
+    (ripple_compress_layers) as soon as it has landed, while the next one is
+    copied, and the decode outputs go back in four parts behind the decode
+    steps."""
+    wl, R = st.wl, st.R
+    L = wl.n_layers
+
     def pin(t):
         h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
         h.copy_(t)
@@ -847,26 +855,56 @@ def measure_e2e(st, args, torch, tokens):
     hq = [pin(t) for t in st.q_win]
     hk = [pin(t) for t in st.k]
     hv = [pin(t) for t in st.v]
-    hdq = [pin(t) for t in st.dq]
-    hdk = [pin(t) for t in st.dk]
-    hdv = [pin(t) for t in st.dv]
+    hd = [pin(t) for t in (st.dq_all, st.dk_all, st.dv_all)]
     hout = torch.empty(st.out.shape, dtype=st.out.dtype).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv + hdq + hdk + hdv)
+    h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv + hd)
     d2h = hout.numel() * hout.element_size()
+    groups = [(g, min(L, g + group)) for g in range(0, L, group)]
+    tables = [R.CompressTables(st.q_win[a:b], st.k[a:b], st.v[a:b], st.k_out[a:b],
+                               st.v_out[a:b], st.idx[a:b]) for a, b in groups]
+    main, side = torch.cuda.current_stream(), torch.cuda.Stream()
+    landed = [torch.cuda.Event() for _ in groups]
+    dec_in, start = torch.cuda.Event(), torch.cuda.Event()
+    parts = [(t, min(wl.decode_steps, t + (wl.decode_steps + 3) // 4))
+             for t in range(0, wl.decode_steps, (wl.decode_steps + 3) // 4)]
+    done = [torch.cuda.Event() for _ in parts]
 
     def step():
-        for layer in range(wl.n_layers):
-            st.q_win[layer].copy_(hq[layer], non_blocking=True)
-            st.k[layer].copy_(hk[layer], non_blocking=True)
-            st.v[layer].copy_(hv[layer], non_blocking=True)
-        for t in range(wl.decode_steps):
-            st.dq[t].copy_(hdq[t], non_blocking=True)
-            st.dk[t].copy_(hdk[t], non_blocking=True)
-            st.dv[t].copy_(hdv[t], non_blocking=True)
-        st.step()
-        hout.copy_(st.out, non_blocking=True)
+        start.record(main)
+        side.wait_event(start)  # the previous step is done with the inputs
+        with torch.cuda.stream(side):
+            st.dq_all.copy_(hd[0], non_blocking=True)
+            st.dk_all.copy_(hd[1], non_blocking=True)
+            st.dv_all.copy_(hd[2], non_blocking=True)
+            dec_in.record(side)
+            for (a, b), ev in zip(groups, landed):
+                for layer in range(a, b):
+                    st.q_win[layer].copy_(hq[layer], non_blocking=True)
+                    st.k[layer].copy_(hk[layer], non_blocking=True)
+                    st.v[layer].copy_(hv[layer], non_blocking=True)
+                ev.record(side)
+        for (a, b), ev, tab in zip(groups, landed, tables):
+            main.wait_event(ev)
+            n = R.ripple_compress_layers(st.desc, st.budgets[a:b], tab, st.ws,
+                                         dev_status=st.status)
+            assert n == st.n_keep[a:b]
+        main.wait_event(dec_in)
+        st.lens.copy_(st.lens0)
+        for (t0, t1), ev in zip(parts, done):
+            for t in range(t0, t1):
+                R.ripple_decode_attn(st.ddesc, st.dq[t], st.dk[t], st.dv[t], st.tables, st.lens,
+                                     st.out[t], st.dws, dev_status=st.status)
+            ev.record(main)
+            side.wait_event(ev)
+            with torch.cuda.stream(side):
+                hout[t0:t1].copy_(st.out[t0:t1], non_blocking=True)
+        main.wait_stream(side)
 
-    step()
+    # freshly pinned buffers copy at a fraction of the link's rate for their
+    # first one or two uses (measured: 124-178 ms, then 83 ms for the same
+    # 17.4 GB), so three untimed steps come first
+    for _ in range(3):
+        step()
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
@@ -877,7 +915,10 @@ def measure_e2e(st, args, torch, tokens):
     torch.cuda.synchronize()
     ms = t0.elapsed_time(t1) / args.e2e_steps
     return {"value": round(tokens / (ms / 1e3), 1), "unit": "tokens/s", "ms_per_step": round(ms, 3),
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+            "warmup_steps": 3,
+            "overlap": f"host->device copies on a second stream, compression per {group} layers "
+                       "as they land, outputs back in four parts behind the decode steps"}
 
 
 # ----------------------------------------------------------------- CPU oracle
