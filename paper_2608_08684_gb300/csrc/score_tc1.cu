@@ -56,7 +56,12 @@ constexpr int kThreads = 352;
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
-constexpr int kMinTilesPerItemO = 9;  // kO: the same, with the values and partials in L2 too
+// kO: items of a third of a 32k unit. Each item's partial output, its
+// row-slice sum and the pass-2 wait on the unit's other items cost more than
+// re-reading the keys from DRAM (an item's keys no longer stay in L2 until
+// its pass 2): 32 layers of the 32k workload took 8.57 ms with 9-tile items,
+// 7.34 / 6.83 / 6.22 / 6.42 ms with 48 / 64 / 86 / 128.
+constexpr int kMinTilesPerItemO = 86;
 constexpr int kMaxStages = 4;
 constexpr int kOReduceLag = 2;  // kO: a step's item rows are summed this many steps later
 
