@@ -169,6 +169,7 @@ struct Misc {
   // between the warpgroups, but not strictly across a step's pass-1 tiles, and
   // a parity wait only tells apart phases one apart), and the O accumulator
   uint64_t p_full[2], p_empty[2], o_full, o_empty;
+  float vhalf[2][128];  // kO: warpgroup 1's half of each key's vote, per tile parity
   uint32_t tmem_base;
   int abort_flag;
   long long wait_cycles;  // bound of the waits of this launch
@@ -187,6 +188,13 @@ struct Tc1Smem {
   static constexpr int Bytes = OffMisc + (int)sizeof(Misc) + 1024;  // + alignment slack
   static_assert(Bytes <= 227 * 1024, "shared memory budget");
 };
+
+// count arrivals on a barrier at once
+__device__ __forceinline__ void mbar_arrive_cnt(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(count)
+               : "memory");
+}
 
 __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, Misc *ms,
                                          int32_t *status) {
@@ -271,27 +279,72 @@ __device__ __forceinline__ void oseq_at(const Step &s, int j, int &kind, int &id
   }
 }
 
-// Probabilities of one key (this thread's TMEM lane) for the 128 window rows,
-// as bf16 pairs (rows 2i and 2i + 1 in pk[i]), into the shared-memory tile in
-// the MN-major, 128-byte-swizzled layout the tensor core reads as the A
-// operand of O = P . V: rows 0-63 and 64-127 in two 16 KB halves, in each the
-// key's 128-byte line holds its 64 rows, 16-byte chunk c at position
-// c ^ (key mod 8).
-__device__ __forceinline__ void store_p_row(uint8_t *ptile, int key, const uint32_t (&pk)[64]) {
-#pragma unroll
-  for (int half = 0; half < 2; ++half)
-#pragma unroll
-    for (int c = 0; c < 8; ++c) {
-      const int w = half * 32 + c * 4;  // rows 8c .. 8c + 7 of the half
-      uint8_t *dst = ptile + half * kHalfBytes + (key >> 3) * 1024 + (key & 7) * 128 +
-                     ((c ^ (key & 7)) << 4);
-      *reinterpret_cast<uint4 *>(dst) = make_uint4(pk[w], pk[w + 1], pk[w + 2], pk[w + 3]);
-    }
-}
-
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   const __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<const uint32_t *>(&b);
+}
+
+// Probabilities of this thread's key for 64 window rows (logit columns
+// c0 * 32 .. c0 * 32 + 63 of a pass-2 tile, x = those columns) and their sum
+// in a fixed order; with kP also as bf16 pairs (rows 2i, 2i + 1 of the 64 in
+// pk[i]), zero for the rows a window key is hidden from (hidden_below: the
+// rows of window position below it; -1 for a prefix key). A key's vote is
+// the sum of its two halves, half 0 + half 1, in every mode.
+template <bool kP>
+__device__ __forceinline__ float half_probs(const uint32_t (&x)[2][32], const float4 *o4, int c0,
+                                            float scale2, int hidden_below, int W,
+                                            uint32_t (&pk)[32]) {
+  // fp32x2: logits scaled and shifted two at a time, sums in pairs
+  float2 sv[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
+  const float2 s2 = make_float2(scale2, scale2);
+#pragma unroll
+  for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+    for (int j4 = 0; j4 < 8; ++j4) {
+      const int c = c0 + cc;
+      const float4 o = o4[c * 8 + j4];
+      const float2 y0 = __ffma2_rn(make_float2(__uint_as_float(x[cc][4 * j4]),
+                                               __uint_as_float(x[cc][4 * j4 + 1])),
+                                   s2, make_float2(-o.x, -o.y));
+      const float2 y1 = __ffma2_rn(make_float2(__uint_as_float(x[cc][4 * j4 + 2]),
+                                               __uint_as_float(x[cc][4 * j4 + 3])),
+                                   s2, make_float2(-o.z, -o.w));
+      float2 e0 = make_float2(fast_exp2(y0.x), fast_exp2(y0.y));
+      float2 e1 = make_float2(fast_exp2(y1.x), fast_exp2(y1.y));
+      if constexpr (kP) {
+        if (hidden_below >= 0) {
+          const int col = c * 32 + 4 * j4;  // window row of e0.x
+          if ((col + 0) % W < hidden_below) e0.x = 0.f;
+          if ((col + 1) % W < hidden_below) e0.y = 0.f;
+          if ((col + 2) % W < hidden_below) e1.x = 0.f;
+          if ((col + 3) % W < hidden_below) e1.y = 0.f;
+        }
+        pk[(cc * 32 + 4 * j4) >> 1] = pack_bf16x2(e0.x, e0.y);
+        pk[((cc * 32 + 4 * j4) >> 1) + 1] = pack_bf16x2(e1.x, e1.y);
+      }
+      sv[(2 * j4) & 3] = __fadd2_rn(sv[(2 * j4) & 3], e0);
+      sv[(2 * j4 + 1) & 3] = __fadd2_rn(sv[(2 * j4 + 1) & 3], e1);
+    }
+  return ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) + ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
+}
+
+// Half h (window rows 64h .. 64h + 63) of one key's probabilities (this
+// thread's TMEM lane), as bf16 pairs (rows 2i and 2i + 1 of the half in
+// pk[i]), into the shared-memory tile in the MN-major, 128-byte-swizzled
+// layout the tensor core reads as the A operand of O = P . V: rows 0-63 and
+// 64-127 in two 16 KB halves, in each the key's 128-byte line holds its 64
+// rows, 16-byte chunk c at position c ^ (key mod 8).
+__device__ __forceinline__ void store_p_half(uint8_t *ptile, int key, int h,
+                                             const uint32_t (&pk)[32]) {
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const int w = c * 4;  // rows 8c .. 8c + 7 of the half
+    uint8_t *dst = ptile + h * kHalfBytes + (key >> 3) * 1024 + (key & 7) * 128 +
+                   ((c ^ (key & 7)) << 4);
+    *reinterpret_cast<uint4 *>(dst) = make_uint4(pk[w], pk[w + 1], pk[w + 2], pk[w + 3]);
+  }
 }
 
 // kO: the output rows of item `it`'s slice of its unit (rows chunk * 128 /
@@ -363,7 +416,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&ms->q_empty, 1);
     for (int i = 0; i < C::NA; ++i) {
       mbar_init(&ms->acc_full[i], 1);
-      mbar_init(&ms->acc_empty[i], 4);
+      // kO: pass-2 tiles are released by all eight epilogue warps, pass-1
+      // tiles by the four of their warpgroup with two arrivals each
+      mbar_init(&ms->acc_empty[i], kO ? 8 : 4);
     }
     mbar_init(&ms->qs_full, 1);
     mbar_init(&ms->qs_empty, 1);
@@ -373,7 +428,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&ms->mma_done, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&ms->p_full[i], 4);
+      mbar_init(&ms->p_full[i], 8);
       mbar_init(&ms->p_empty[i], 1);
     }
     mbar_init(&ms->o_full, 1);
@@ -464,10 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ MMA issuer
     if (lane == 0) {
       int kcount = 0, acount = 0, qcount = 0, ocount = 0;
-      // kO: bit s mod 4 = the warpgroup that writes pass-2 tile s's
-      // probabilities; tiles consumed per writing warpgroup
-      uint32_t pv_owner = 0;
-      int pv_count0 = 0, pv_count1 = 0;
+      int pv_count = 0;  // kO: probability tiles multiplied
       constexpr uint32_t id = idesc_bf16(128, 128);
       // O = P . V: P (rows x keys) and V (keys x dims) both MN-major
       constexpr uint32_t id_pv = idesc_bf16(128, 128) | (1u << 15) | (1u << 16);
@@ -493,11 +545,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // O (+)= P . V for pass-2 tile s, once the epilogue has written
             // its probabilities (and, for the item's first tile, has read
             // out the previous item's O)
-            static_assert(kPvLag + 2 <= 32, "owner bits");
-            const int ow = (pv_owner >> (s % (kPvLag + 2))) & 1;
-            const int pvc = ow ? pv_count1 : pv_count0;
             if ((s == 0 && !wait_bar(&ms->o_empty, (ocount & 1) ^ 1, ms, p.status)) ||
-                !wait_bar(&ms->p_full[ow], pvc & 1, ms, p.status) ||
+                !wait_bar(&ms->p_full[0], pv_count & 1, ms, p.status) ||
                 !wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status)) {
               ok = false;
               break;
@@ -508,12 +557,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(tmem + C::OCol, sw128_desc_mn(pbase + kk * 2048, kHalfBytes, 1024),
                        sw128_desc_mn(ka + kk * 2048, kHalfBytes, 1024), id_pv, kk > 0 || s > 0);
             mma_commit(&ms->k_empty[ks]);
-            mma_commit(&ms->p_empty[ow]);
+            mma_commit(&ms->p_empty[0]);
             ++kcount;
-            if (ow)
-              ++pv_count1;
-            else
-              ++pv_count0;
+            ++pv_count;
             if (s == st.n2 - 1) {
               mma_commit(&ms->o_full);
               ++ocount;
@@ -528,10 +574,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           const int as = acount % C::NA;
-          if (kO && kind == 2) {
-            const uint32_t bit = 1u << (s % (kPvLag + 2));
-            pv_owner = wg_of(acount) ? pv_owner | bit : pv_owner & ~bit;
-          }
           if (!wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status) ||
               !wait_bar(&ms->acc_empty[as], ((acount / C::NA) & 1) ^ 1, ms, p.status)) {
             ok = false;
@@ -635,8 +677,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(quarter * 32) << 16;
     int tcount = 0;  // tiles seen
     int oc = 0;            // kO: pass-2 items seen
-    int pw0 = 0, pw1 = 0;  // kO: probability tiles written, per warpgroup
-    int prev_writer = -1;  // kO: the warpgroup that wrote the previous tile
+    int ptc = 0;           // kO: probability tiles written
 
     // Inside an item every warp follows the same control flow even if a wait
     // gives up (the tile is then skipped), so that the named barriers below
@@ -662,7 +703,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_wait_ld();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+            if (lane == 0) mbar_arrive_cnt(&ms->acc_empty[as], kO ? 2 : 1);
             if ((t + 1) * kTile - 1 >= p.P) {  // keys this row cannot see -> -inf
 #pragma unroll
               for (int c = 0; c < 4; ++c)
@@ -724,10 +765,44 @@ __global__ void __launch_bounds__(kThreads, 1)
             named_bar_sync(3 + wg, 128);
           }
           const int t = st.b0 + s;
-          const int mine = wg_of(tcount) == wg;
           const int as = tcount % C::NA, ph = (tcount / C::NA) & 1;
-          ++tcount;
-          if (mine && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
+          if constexpr (kO) {
+            const int key = t * kTile + r;
+            // both warpgroups take every pass-2 tile, each for 64 of its 128
+            // window rows (logit columns 64 wg ..): its half of the key's
+            // probabilities, half of the vote (summed over the warpgroups
+            // through shared memory) and its half of the probability tile
+            const bool got = warp_wait(&ms->acc_full[as], ph, ms, p.status);
+            float half = 0.f;
+            if (got) {
+              tc_fence_after();
+              uint32_t x[2][32];
+              tmem_ld32(tmem + lane_addr + as * 128 + wg * 64, x[0]);
+              tmem_ld32(tmem + lane_addr + as * 128 + wg * 64 + 32, x[1]);
+              tmem_wait_ld();
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
+              // a window key (or a key past the end) is seen only by the rows
+              // at or after it (causal inside the window)
+              uint32_t pk[32];
+              half = half_probs<true>(x, reinterpret_cast<const float4 *>(ms->offs[wg]), 2 * wg,
+                                      p.scale2, key >= p.P ? key - p.P : -1, p.W, pk);
+              // into the tile once the previous tile's probabilities have
+              // been multiplied
+              if (ptc > 0) warp_wait(&ms->p_empty[0], (ptc - 1) & 1, ms, p.status);
+              store_p_half(ptile, r, wg, pk);
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&ms->p_full[0]);
+            }
+            if (wg == 1) ms->vhalf[ptc & 1][r] = half;
+            named_bar_sync(6, 256);
+            if (wg == 0 && got && key < p.P)
+              p.votes[guard((long long)st.u2 * p.P + key, 1, (long long)p.units * p.P, p.status)] =
+                  half + ms->vhalf[ptc & 1][r];
+            ++ptc;
+          } else if (wg_of(tcount) == wg && warp_wait(&ms->acc_full[as], ph, ms, p.status)) {
             tc_fence_after();
             uint32_t x[4][32];
 #pragma unroll
@@ -736,17 +811,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&ms->acc_empty[as]);
-            // fp32x2: logits scaled and shifted two at a time, sums in pairs
-            float2 sv[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) sv[i] = make_float2(0.f, 0.f);
-            const float2 s2 = make_float2(p.scale2, p.scale2);
             const float4 *o4 = reinterpret_cast<const float4 *>(ms->offs[wg]);
-            const int key = t * kTile + r;
-            // kO: a window key (or a key past the end) is seen only by the
-            // rows at or after it (causal inside the window)
-            const int hidden_below = kO && key >= p.P ? key - p.P : -1;
-            uint32_t pk[kO ? 64 : 1];  // kO: the probabilities as bf16 pairs
+            // the two halves' sums as half_probs forms them, in one pass
+            float2 sv[2][4];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) sv[i >> 2][i & 3] = make_float2(0.f, 0.f);
+            const float2 s2 = make_float2(p.scale2, p.scale2);
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
@@ -758,50 +828,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float2 y1 = __ffma2_rn(make_float2(__uint_as_float(x[c][4 * j4 + 2]),
                                                          __uint_as_float(x[c][4 * j4 + 3])),
                                              s2, make_float2(-o.z, -o.w));
-                float2 e0 = make_float2(fast_exp2(y0.x), fast_exp2(y0.y));
-                float2 e1 = make_float2(fast_exp2(y1.x), fast_exp2(y1.y));
-                if constexpr (kO) {
-                  if (hidden_below >= 0) {
-                    const int col = c * 32 + 4 * j4;  // window row of e0.x
-                    if ((col + 0) % p.W < hidden_below) e0.x = 0.f;
-                    if ((col + 1) % p.W < hidden_below) e0.y = 0.f;
-                    if ((col + 2) % p.W < hidden_below) e1.x = 0.f;
-                    if ((col + 3) % p.W < hidden_below) e1.y = 0.f;
-                  }
-                  pk[(c * 32 + 4 * j4) >> 1] = pack_bf16x2(e0.x, e0.y);
-                  pk[((c * 32 + 4 * j4) >> 1) + 1] = pack_bf16x2(e1.x, e1.y);
-                }
-                sv[(2 * j4) & 3] = __fadd2_rn(sv[(2 * j4) & 3], e0);
-                sv[(2 * j4 + 1) & 3] = __fadd2_rn(sv[(2 * j4 + 1) & 3], e1);
+                float2 *h = sv[c >> 1];
+                h[(2 * j4) & 3] =
+                    __fadd2_rn(h[(2 * j4) & 3], make_float2(fast_exp2(y0.x), fast_exp2(y0.y)));
+                h[(2 * j4 + 1) & 3] = __fadd2_rn(h[(2 * j4 + 1) & 3],
+                                                 make_float2(fast_exp2(y1.x), fast_exp2(y1.y)));
               }
-            const float vote = ((sv[0].x + sv[0].y) + (sv[1].x + sv[1].y)) +
-                               ((sv[2].x + sv[2].y) + (sv[3].x + sv[3].y));
-            if constexpr (kO) {
-              // this key's probabilities of the 128 rows into the tile the
-              // MMA warp multiplies by the value tile, once it has read the
-              // previous tile's
-              // once the previous tile's probabilities have been multiplied
-              // (its writer's pw[.] - 1-th phase)
-              if (prev_writer >= 0)
-                warp_wait(&ms->p_empty[prev_writer], ((prev_writer ? pw1 : pw0) - 1) & 1, ms,
-                          p.status);
-              store_p_row(ptile, r, pk);
-              fence_proxy_async_smem();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(&ms->p_full[wg]);
-            }
+            const float h0 = ((sv[0][0].x + sv[0][0].y) + (sv[0][1].x + sv[0][1].y)) +
+                             ((sv[0][2].x + sv[0][2].y) + (sv[0][3].x + sv[0][3].y));
+            const float h1 = ((sv[1][0].x + sv[1][0].y) + (sv[1][1].x + sv[1][1].y)) +
+                             ((sv[1][2].x + sv[1][2].y) + (sv[1][3].x + sv[1][3].y));
+            const int key = t * kTile + r;
             if (key < p.P)
               p.votes[guard((long long)st.u2 * p.P + key, 1, (long long)p.units * p.P, p.status)] =
-                  vote;
+                  h0 + h1;
           }
-          if (kO) {
-            const int writer = wg_of(tcount - 1);
-            if (writer)
-              ++pw1;
-            else
-              ++pw0;
-            prev_writer = writer;
-          }
+          ++tcount;
         }
       }
       if (kO && st.n2 > 0) {
