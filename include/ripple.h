@@ -233,11 +233,16 @@ ripple_status ripple_compress_layers_attn_workspace_bytes(const ripple_layer_des
  *             [B][Hq][w][head_dim], 16-byte aligned, written
  * workspace   at least ripple_compress_layers_attn_workspace_bytes bytes,
  *             256-byte aligned, no initialisation needed
- * Other arguments, outputs and errors as ripple_compress_layers; the kept
- * counts, indices and gathered rows equal that call's bit for bit. o_win is
- * accumulated in fp32 from bf16 probabilities (the tensor cores' operand
- * type) in a fixed order: the same on every run. The call may be captured in a
- * CUDA graph.
+ * Other arguments, outputs and errors as ripple_compress_layers, with the same
+ * kept counts. The two calls split a unit's keys into different items (this
+ * one takes up to 32768 keys a unit as one), so the row normalisers, merged
+ * from the items' partial statistics, can differ in their last bits, and a
+ * token whose pooled vote ties the selection threshold to within that
+ * rounding can be kept by one call and not the other; units of at most 1152
+ * keys are one item in both, and then the indices and gathered rows are
+ * equal bit for bit. o_win is accumulated in fp32 from bf16 probabilities
+ * (the tensor cores' operand type) in a fixed order: the same on every run.
+ * The call may be captured in a CUDA graph.
  */
 ripple_status ripple_compress_layers_attn(const ripple_layer_desc *desc, int32_t n_layers,
                                           const int64_t *budgets_host,

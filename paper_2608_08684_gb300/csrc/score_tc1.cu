@@ -26,8 +26,10 @@
 // prefill attention of the window rows, so that a real prefill reads the keys
 // for both in one pass): pass 2 covers every key, causal inside the window;
 // the producer streams each value tile behind the next key tile through the
-// same ring (three stages); the epilogue writes the tile's probabilities as
-// bf16 into a shared-memory tile (MN-major, the A operand) and the MMA warp
+// same ring (three stages); both epilogue warpgroups take every pass-2 tile,
+// each for 64 of its 128 window rows, and write those rows' probabilities as
+// bf16 into a shared-memory tile (MN-major, the A operand; a key's vote is
+// its two halves summed through shared memory), and the MMA warp
 // accumulates O[row][dim] += P . V in the last 128 TMEM columns (V, MN-major,
 // the B operand). The probabilities are final (pass 1 has fixed every row's
 // normaliser), so O needs no rescaling. At an item's end both warpgroups
@@ -56,12 +58,12 @@ constexpr int kThreads = 352;
 constexpr int kLag = 1;                         // pass 2 of item k runs in step k + kLag
 constexpr int kPubSlots = 2;
 constexpr int kMinTilesPerItem = 9;
-// kO: items of a third of a 32k unit. Each item's partial output, its
-// row-slice sum and the pass-2 wait on the unit's other items cost more than
-// re-reading the keys from DRAM (an item's keys no longer stay in L2 until
-// its pass 2): 32 layers of the 32k workload took 8.57 ms with 9-tile items,
-// 7.34 / 6.83 / 6.22 / 6.42 ms with 48 / 64 / 86 / 128.
-constexpr int kMinTilesPerItemO = 86;
+// kO: a whole unit per item up to 32768 keys. An item's partial output, its
+// row-slice sum and pass 2's wait on the unit's other items cost more than
+// re-reading the keys from DRAM in pass 2 (an item's keys no longer stay in
+// L2 until then): 32 layers of the 32k workload took 5.39 / 5.25 / 5.08 /
+// 5.11 / 5.00 ms with items of 32 / 64 / 86 / 128 / 256 tiles.
+constexpr int kMinTilesPerItemO = 256;
 constexpr int kMaxStages = 4;
 constexpr int kOReduceLag = 2;  // kO: a step's item rows are summed this many steps later
 

@@ -171,7 +171,7 @@ def test_compress_layers_attn_checked(lib, chk):
     # the scoring fused into the window rows' prefill attention (several items
     # per unit, window keys across the last tiles)
     wl = synth.WORKLOADS["tiny"].replace(n_layers=2, batch=1, n_q_heads=8, n_kv_heads=2,
-                                         head_dim=128, seq_len=12000, dtype="bf16", seed=68)
+                                         head_dim=128, seq_len=33000, dtype="bf16", seed=68)
     budgets = [300, 1500]
     B, H, d = wl.batch, wl.n_kv_heads, wl.head_dim
     ins = [tuple(t.to(DEV) for t in C.layer_inputs(wl, l, "cpu")) for l in range(wl.n_layers)]

@@ -95,8 +95,8 @@ SHAPES = [
     ("G4-T132", dict(n_layers=1, batch=1, n_q_heads=4, n_kv_heads=1, head_dim=128, seq_len=132,
                      dtype="bf16", seed=82), [60]),
     # two items per unit (the partial outputs summed in item order)
-    ("G4-T12000", dict(n_layers=2, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
-                       seq_len=12000, dtype="bf16", kv_dist="scaled_sinks", seed=83),
+    ("G4-T33000", dict(n_layers=2, batch=1, n_q_heads=8, n_kv_heads=2, head_dim=128,
+                       seq_len=33000, dtype="bf16", kv_dist="scaled_sinks", seed=83),
      [700, 10**6]),
     # G 8, w 16
     ("G8-w16", dict(n_layers=2, batch=1, n_q_heads=16, n_kv_heads=2, head_dim=128, seq_len=777,
