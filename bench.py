@@ -121,14 +121,16 @@ def run_case(args):
         idx = torch.empty(B * Hkv * n, dtype=torch.int32, device=dev)
         nbytes = B * Hkv * d * e * (wl.seq_len + 3 * n) + B * Hq * wl.window * d * e
         if args.layers > 1:
-            # several layers in one call: the budgets of the args.layers
-            # largest-budget layers, every layer reading the same K/V
+            # several layers in one call: the args.layers largest-budget
+            # layers, each with its own inputs
             lay = sorted(range(L), key=lambda i: -budgets[i])[:args.layers]
             outs = [(torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
                      torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
                      torch.empty(B * Hkv * n_keep[i], dtype=torch.int32, device=dev))
                     for i in lay]
-            tabs = R.CompressTables([q_win] * len(lay), [k] * len(lay), [v] * len(lay),
+            ins = [(synth.layer_window_queries(wl, i, dev), synth.layer_keys(wl, i, dev),
+                    synth.layer_values(wl, i, dev)) for i in lay]
+            tabs = R.CompressTables([x[0] for x in ins], [x[1] for x in ins], [x[2] for x in ins],
                                     [o[0] for o in outs], [o[1] for o in outs],
                                     [o[2] for o in outs])
             ws = torch.empty(R.ripple_compress_layers_workspace_bytes(desc, len(lay)),
@@ -147,8 +149,8 @@ def run_case(args):
             b_.record()
             if i >= 2:
                 times.append((a, b_))
-        what = (f"compress {len(lay)} layers in one call (budgets of layers {lay}, K/V of "
-                f"layer {layer})" if args.layers > 1 else
+        what = (f"compress {len(lay)} layers in one call (layers {lay}, each with its own "
+                f"inputs)" if args.layers > 1 else
                 f"compress layer {layer} (budget {budgets[layer]}, n {n})")
     else:
         steps = args.repeat
@@ -201,7 +203,7 @@ def run_attn_case(args, R, synth, wl, dev, budgets, n_keep):
 def attn_measure(R, synth, wl, dev, budgets, n_keep, n_layers, repeat):
     """The scoring fused into the prefill attention of the window rows
     (ripple_compress_layers_attn) on the n_layers largest-budget layers in
-    one call (every layer reading the same K/V, inputs above L2), beside
+    one call (each layer with its own inputs, above L2), beside
     ripple_compress_layers on the same inputs. Algorithmic bytes of the fused
     call: the compression's, plus V read in full and the fp32 outputs. The
     separate alternative would read the window rows' K and V once more (the
@@ -212,17 +214,16 @@ def attn_measure(R, synth, wl, dev, budgets, n_keep, n_layers, repeat):
                            wl.elem_bytes)
     nl = max(1, min(n_layers, L))
     lay = sorted(range(L), key=lambda i: -budgets[i])[:nl]
-    layer = lay[0]
-    q_win = synth.layer_window_queries(wl, layer, dev)
-    k = synth.layer_keys(wl, layer, dev)
-    v = synth.layer_values(wl, layer, dev)
     desc = R.layer_desc(B, Hq, Hkv, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
                         wl.torch_dtype)
     outs = [(torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
              torch.empty(B, Hkv, n_keep[i], d, dtype=wl.torch_dtype, device=dev),
              torch.empty(B * Hkv * n_keep[i], dtype=torch.int32, device=dev)) for i in lay]
-    tabs = R.CompressTables([q_win] * nl, [k] * nl, [v] * nl, [o[0] for o in outs],
-                            [o[1] for o in outs], [o[2] for o in outs])
+    # every layer its own inputs: layers reading one K/V would share it in L2
+    ins = [(synth.layer_window_queries(wl, i, dev), synth.layer_keys(wl, i, dev),
+            synth.layer_values(wl, i, dev)) for i in lay]
+    tabs = R.CompressTables([x[0] for x in ins], [x[1] for x in ins], [x[2] for x in ins],
+                            [o[0] for o in outs], [o[1] for o in outs], [o[2] for o in outs])
     o_win = [torch.empty(B, Hq, wl.window, d, device=dev) for _ in lay]
     ws_a = torch.empty(R.ripple_compress_layers_attn_workspace_bytes(desc, nl), dtype=torch.uint8,
                        device=dev)
@@ -255,7 +256,7 @@ def attn_measure(R, synth, wl, dev, budgets, n_keep, n_layers, repeat):
     gbs = attn_bytes / (ms_a / 1e3) / 1e9
     return {
         "what": (f"compress {nl} layers with the window rows' attention output in one call "
-                 f"(budgets of layers {lay}, K/V of layer {layer})"),
+                 f"(layers {lay}, each with its own inputs)"),
         "calls": repeat, "ms_per_call": round(ms_a, 5), "bytes_per_call": attn_bytes,
         "gbs": round(gbs, 1), "frac_hbm": round(gbs / hbm, 4),
         "compress_only_ms": round(ms_c, 5),
