@@ -167,10 +167,9 @@ struct Misc {
   uint64_t acc_full[kMaxStages], acc_empty[kMaxStages];
   uint64_t qs_full, qs_empty;           // pass-2 queries in shared memory
   uint64_t pub_full[kPubSlots], pub_empty[kPubSlots], mma_done;
-  // kO: the probability tile, per writing warpgroup (the tiles alternate
-  // between the warpgroups, but not strictly across a step's pass-1 tiles, and
-  // a parity wait only tells apart phases one apart), and the O accumulator
-  uint64_t p_full[2], p_empty[2], o_full, o_empty;
+  // kO: the probability tile (all eight epilogue warps write each tile, the
+  // P . V MMA releases it) and the O accumulator
+  uint64_t p_full, p_empty, o_full, o_empty;
   float vhalf[2][128];  // kO: warpgroup 1's half of each key's vote, per tile parity
   uint32_t tmem_base;
   int abort_flag;
@@ -429,10 +428,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ms->pub_empty[i], 1);
     }
     mbar_init(&ms->mma_done, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&ms->p_full[i], 8);
-      mbar_init(&ms->p_empty[i], 1);
-    }
+    mbar_init(&ms->p_full, 8);
+    mbar_init(&ms->p_empty, 1);
     mbar_init(&ms->o_full, 1);
     mbar_init(&ms->o_empty, 8);
     ms->abort_flag = 0;
@@ -548,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // its probabilities (and, for the item's first tile, has read
             // out the previous item's O)
             if ((s == 0 && !wait_bar(&ms->o_empty, (ocount & 1) ^ 1, ms, p.status)) ||
-                !wait_bar(&ms->p_full[0], pv_count & 1, ms, p.status) ||
+                !wait_bar(&ms->p_full, pv_count & 1, ms, p.status) ||
                 !wait_bar(&ms->k_full[ks], (kcount / C::NK) & 1, ms, p.status)) {
               ok = false;
               break;
@@ -559,7 +556,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               mma_bf16(tmem + C::OCol, sw128_desc_mn(pbase + kk * 2048, kHalfBytes, 1024),
                        sw128_desc_mn(ka + kk * 2048, kHalfBytes, 1024), id_pv, kk > 0 || s > 0);
             mma_commit(&ms->k_empty[ks]);
-            mma_commit(&ms->p_empty[0]);
+            mma_commit(&ms->p_empty);
             ++kcount;
             ++pv_count;
             if (s == st.n2 - 1) {
@@ -792,11 +789,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                       p.scale2, key >= p.P ? key - p.P : -1, p.W, pk);
               // into the tile once the previous tile's probabilities have
               // been multiplied
-              if (ptc > 0) warp_wait(&ms->p_empty[0], (ptc - 1) & 1, ms, p.status);
+              if (ptc > 0) warp_wait(&ms->p_empty, (ptc - 1) & 1, ms, p.status);
               store_p_half(ptile, r, wg, pk);
               fence_proxy_async_smem();
               __syncwarp();
-              if (lane == 0) mbar_arrive(&ms->p_full[0]);
+              if (lane == 0) mbar_arrive(&ms->p_full);
             }
             if (wg == 1) ms->vhalf[ptc & 1][r] = half;
             named_bar_sync(6, 256);
