@@ -45,12 +45,19 @@ def _both(lib, wl, budgets, cap_extra=2, device_gen="cpu"):
 
 
 SHAPES = [
-    # tensor-core path (G * w = 128): all layers in three launches
+    # tensor-core path (G * w = 128): all layers in two or three launches
     ("bf16-d128-G4", dict(n_layers=6, batch=2, n_q_heads=8, n_kv_heads=2, head_dim=128,
                           seq_len=1000, dtype="bf16", kv_dist="scaled_sinks", seed=21),
      [0, 31, 32, 200, 968, 10**6]),
     ("bf16-d128-G4-one-tile", dict(n_layers=3, batch=1, n_q_heads=4, n_kv_heads=1,
                                    head_dim=128, seq_len=130, dtype="bf16", seed=22), [40, 98, 129]),
+    # 256 units: the one-CTA-per-unit selection that also gathers (window-only,
+    # keep-all and ragged layers) against the per-layer calls' cluster
+    # selection and gather kernel
+    ("bf16-d128-G4-256-units", dict(n_layers=8, batch=4, n_q_heads=32, n_kv_heads=8,
+                                    head_dim=128, seq_len=1000, dtype="bf16",
+                                    kv_dist="scaled_sinks", seed=25),
+     [0, 31, 32, 200, 500, 968, 999, 10**6]),
     # other shapes: scoring layer by layer, one selection and one gather launch for all layers
     ("bf16-d128-G8", dict(n_layers=3, batch=1, n_q_heads=16, n_kv_heads=2, head_dim=128,
                           seq_len=700, dtype="bf16", seed=23), [300, 50, 699]),
