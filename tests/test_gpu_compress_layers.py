@@ -63,6 +63,14 @@ SHAPES = [
                           seq_len=700, dtype="bf16", seed=23), [300, 50, 699]),
     ("f32-d64-G2", dict(n_layers=4, batch=1, n_q_heads=4, n_kv_heads=2, head_dim=64,
                         seq_len=300, dtype="f32", seed=24), [64, 10, 300, 128]),
+    # 256 units on the CUDA-core scoring path: the gathering selection with
+    # 256-byte fp32 rows and 128-byte bf16 rows
+    ("f32-d64-G2-256-units", dict(n_layers=8, batch=4, n_q_heads=16, n_kv_heads=8,
+                                  head_dim=64, seq_len=300, dtype="f32", seed=26),
+     [10, 32, 64, 100, 150, 268, 299, 10**6]),
+    ("bf16-d64-G2-256-units", dict(n_layers=8, batch=4, n_q_heads=16, n_kv_heads=8,
+                                   head_dim=64, seq_len=300, dtype="bf16", seed=27),
+     [299, 10**6, 10, 150, 32, 64, 100, 268]),
 ]
 
 
