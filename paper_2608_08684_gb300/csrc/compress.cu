@@ -254,18 +254,35 @@ static ripple_status compress_layers_impl(
                                     (const int32_t *const *)idx_out_host, n, k_out_host,
                                     v_out_host, cap, dev_status, st));
   } else {
-    // Other shapes: scoring layer by layer (each layer's votes in its part of
-    // the vote array, the scratch of the multi-layer workspace reused), then
-    // one selection and one gather launch for all layers. A layer that keeps
-    // every token needs no votes (the selection writes 0..T-1 for it).
-    for (int l = 0; l < n_layers; ++l) {
-      if (g.P == 0 || n[l] == g.T) continue;
-      float *votes_l = ws.votes + (size_t)l * g.units * g.P;
-      cudaError_t e = score_tc_supported(g)
-                          ? launch_score_tc(g, q_win_host[l], k_host[l], ws, votes_l, dev_status, st)
-                          : launch_score_simt(g, q_win_host[l], k_host[l], ws, votes_l,
-                                              dev_status, st);
-      RIPPLE_CUDA_TRY(e);
+    // Other shapes: the 256-row tensor-core scoring of every layer that needs
+    // votes in one launch, or the CUDA-core scoring layer by layer (each
+    // layer's votes in its part of the vote array, the scratch of the
+    // multi-layer workspace reused); then one selection and one gather launch
+    // for all layers. A layer that keeps every token needs no votes (the
+    // selection writes 0..T-1 for it).
+    if (g.P > 0 && score_tc_supported(g)) {
+      // the layers that need votes, all in one tensor-core launch
+      int slots[RIPPLE_COMPRESS_MAX_LAYERS];
+      const void *qs[RIPPLE_COMPRESS_MAX_LAYERS];
+      const void *ks[RIPPLE_COMPRESS_MAX_LAYERS];
+      int n_scored = 0;
+      for (int l = 0; l < n_layers; ++l) {
+        if (n[l] == g.T) continue;
+        slots[n_scored] = l;
+        qs[n_scored] = q_win_host[l];
+        ks[n_scored] = k_host[l];
+        ++n_scored;
+      }
+      if (n_scored > 0)
+        RIPPLE_CUDA_TRY(launch_score_tc(g, n_layers, slots, n_scored, qs, ks, ws, ws.votes,
+                                        dev_status, st));
+    } else {
+      for (int l = 0; l < n_layers; ++l) {
+        if (g.P == 0 || n[l] == g.T) continue;
+        float *votes_l = ws.votes + (size_t)l * g.units * g.P;
+        RIPPLE_CUDA_TRY(launch_score_simt(g, q_win_host[l], k_host[l], ws, votes_l, dev_status,
+                                          st));
+      }
     }
     RIPPLE_CUDA_TRY(launch_select(g, n_layers, ws.votes, ws, n, idx_out_host, dev_status, st,
                                   &ga, &gathered));

@@ -54,6 +54,12 @@ bool score_tc_supported(const LayerGeom &g);
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
                             const CompressWs &ws, float *votes, int32_t *status,
                             cudaStream_t st);
+// The same for n_scored layers of one shape in one launch: scored layer i
+// (q_win[i], k[i]) writes the votes of layer slots[i] of votes
+// [n_slots][g.units][P]; ws is carved for n_scored * g.units units or more.
+cudaError_t launch_score_tc(const LayerGeom &g, int n_slots, const int *slots, int n_scored,
+                            const void *const *q_win, const void *const *k, const CompressWs &ws,
+                            float *votes, int32_t *status, cudaStream_t st);
 // Scoring on the tensor cores for G * w = 128 window rows (bf16, d = 128),
 // for n_layers layers of the same shape in one launch; ws is carved for
 // n_layers * g.units units and votes is [n_layers][g.units][P]. With v (the

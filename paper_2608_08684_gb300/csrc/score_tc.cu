@@ -34,6 +34,8 @@
 #include <cuda.h>
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "kernels.cuh"
 #include "tc_ptx.cuh"
@@ -52,14 +54,16 @@ constexpr int kMinTilesPerItem = 14;
 // ------------------------------------------------------------ work list
 
 struct TcParams {
-  int units, T, P, W, Hq, Hkv, G;
+  int units, upl, T, P, W, Hq, Hkv, G;  // units of all scored layers, units per layer
   int n_tiles1, n_tiles2;  // key tiles of pass 1 (all keys) and pass 2 (prefix keys)
   int tpi, n_ch;           // key tiles per item, items per unit
   int total_items;
   float scale2;
   float2 *partial;  // [units][n_ch][R] (max, sum) per item and row, log2 domain
   float *lognorm;   // [units][R]
-  float *votes;     // [units][P]
+  float *votes;     // [n_layers][upl][P]: unit u's votes at layer_of[u / upl]
+  int layer_of[kCompressMaxLayers];  // the layer (votes slot) of each scored layer
+  int n_slots;                       // layers (votes slots) of the votes array
   int *ctrl;        // [u] items of unit u published; [units + u] row statistics ready
   int32_t *status;
   long long wait_cycles;  // bound of the in-kernel waits
@@ -168,11 +172,20 @@ __device__ __forceinline__ void combine(float &m, float &l, float m2, float l2) 
 
 // ------------------------------------------------------------ kernel
 
+// Kernel argument: the keys of every scored layer as 3-D tensor maps
+// [unit][T][128], their window queries as 2-D maps [B * Hq * W][128], and the
+// parameters.
+struct TcLaunch {
+  CUtensorMap kmap[kCompressMaxLayers];
+  CUtensorMap qmap[kCompressMaxLayers];
+  TcParams p;
+};
+
 template <int NR>
 __global__ void __launch_bounds__(kThreads, 1)
-    score_tc_kernel(const __grid_constant__ CUtensorMap kmap,
-                    const __grid_constant__ CUtensorMap qmap, const __grid_constant__ TcParams p) {
+    score_tc_kernel(const __grid_constant__ TcLaunch lp) {
   using C = Cfg<NR>;
+  const TcParams &p = lp.p;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t *ktiles = smem + C::OFF_K;
@@ -238,8 +251,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
             uint8_t *kb = ktiles + ks * kTileBytes;
             const uint64_t pol = pass == 1 ? keep : drop;
-            tma_load_3d(kb, &kmap, 0, t * kTile, it.unit, &ms->k_full[ks], pol);
-            tma_load_3d(kb + kHalfBytes, &kmap, 64, t * kTile, it.unit, &ms->k_full[ks], pol);
+            const CUtensorMap *km = &lp.kmap[it.unit / p.upl];
+            const int local = it.unit % p.upl;
+            tma_load_3d(kb, km, 0, t * kTile, local, &ms->k_full[ks], pol);
+            tma_load_3d(kb + kHalfBytes, km, 64, t * kTile, local, &ms->k_full[ks], pol);
             ++kcount;
           }
         }
@@ -252,15 +267,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       int qcount = 0;
       for (int k = 0; k < n; ++k) {
         const ItemRef it = item_of(p, k);
-        const int b = it.unit / p.Hkv, h = it.unit % p.Hkv;
+        const int local = it.unit % p.upl;
+        const int b = local / p.Hkv, h = local % p.Hkv;
         const int qrow0 = (b * p.Hq + h * p.G) * p.W;
+        const CUtensorMap *qm = &lp.qmap[it.unit / p.upl];
         const int qs = k % C::NQ;
         if (!wait_bar(&ms->q_empty[qs], ((k / C::NQ) & 1) ^ 1, ms, p.status)) break;
         mbar_arrive_expect_tx(&ms->q_full[qs], C::QBYTES);
         uint8_t *qb = qbufs + qs * C::QBYTES;
         for (int half = 0; half < 2; ++half)
           for (int nr = 0; nr < NR; ++nr)
-            tma_load_2d(qb + half * (NR * kHalfBytes) + nr * kHalfBytes, &qmap, half * 64,
+            tma_load_2d(qb + half * (NR * kHalfBytes) + nr * kHalfBytes, qm, half * 64,
                         qrow0 + nr * 128, &ms->q_full[qs]);
         ++qcount;
       }
@@ -492,6 +509,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           named_bar_sync(3 + wg, 128);
         }
         const float4 *off4 = (const float4 *)ms->off[wg];
+        // the unit's votes slot: its layer's in the vote array
+        const int vunit = p.layer_of[it.unit / p.upl] * p.upl + it.unit % p.upl;
         for (int t = t0; t < t1; ++t, ++tcount) {
           if ((tcount & 1) != wg) continue;
           const int as = tcount % C::NA;
@@ -534,8 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                              ((vs[2].x + vs[2].y) + (vs[3].x + vs[3].y));
           const int key = t * kTile + lrow;
           if (key < p.P)
-            p.votes[guard((long long)it.unit * p.P + key, 1, (long long)p.units * p.P, p.status)] =
-                vote;
+            p.votes[guard((long long)vunit * p.P + key, 1, (long long)p.n_slots * p.upl * p.P,
+                          p.status)] = vote;
         }
       }
     }
@@ -578,34 +597,37 @@ int sm_count() {
 }
 
 template <int NR>
-cudaError_t launch_nr(const LayerGeom &g, const void *q_win, const void *k, const CompressWs &ws,
+cudaError_t launch_nr(const LayerGeom &g, int n_slots, const int *slots, int n_scored,
+                      const void *const *q_win, const void *const *k, const CompressWs &ws,
                       float *votes, int32_t *status, cudaStream_t st) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return cudaErrorNotSupported;
-  CUtensorMap kmap, qmap;
-  {
+  if (n_scored < 1 || n_scored > kCompressMaxLayers || n_slots < 1) return cudaErrorInvalidValue;
+  static TcLaunch lp;  // large: kept off the stack, filled under the lock
+  static std::mutex mu;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int l = 0; l < n_scored; ++l) {
     cuuint64_t dims[3] = {128, (cuuint64_t)g.T, (cuuint64_t)g.units};
     cuuint64_t strides[2] = {256, (cuuint64_t)g.T * 256};
     cuuint32_t box[3] = {64, 128, 1};
     cuuint32_t es[3] = {1, 1, 1};
-    if (enc(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k), dims, strides, box,
-            es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    if (enc(&lp.kmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(k[l]), dims,
+            strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
-  }
-  {
-    cuuint64_t dims[2] = {128, (cuuint64_t)g.B * g.Hq * g.W};
-    cuuint64_t strides[1] = {256};
-    cuuint32_t box[2] = {64, 128};
-    cuuint32_t es[2] = {1, 1};
-    if (enc(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(q_win), dims, strides,
-            box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    cuuint64_t qdims[2] = {128, (cuuint64_t)g.B * g.Hq * g.W};
+    cuuint64_t qstrides[1] = {256};
+    cuuint32_t qbox[2] = {64, 128};
+    cuuint32_t qes[2] = {1, 1};
+    if (enc(&lp.qmap[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(q_win[l]), qdims,
+            qstrides, qbox, qes, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
   const int sms = sm_count();
-  TcParams p;
-  p.units = g.units;
+  TcParams &p = lp.p;
+  p.upl = g.units;
+  p.units = g.units * n_scored;
   p.T = g.T;
   p.P = g.P;
   p.W = g.W;
@@ -620,15 +642,20 @@ cudaError_t launch_nr(const LayerGeom &g, const void *q_win, const void *k, cons
   const int tpi_min = (p.n_tiles1 + sms - 1) / sms;
   p.tpi = tpi_min > kMinTilesPerItem ? tpi_min : kMinTilesPerItem;
   p.n_ch = (p.n_tiles1 + p.tpi - 1) / p.tpi;
-  p.total_items = g.units * p.n_ch;
+  p.total_items = p.units * p.n_ch;
   p.scale2 = g.scale2;
   p.partial = ws.row_partial;
   p.lognorm = ws.row_lognorm;
   p.votes = votes;
+  for (int l = 0; l < n_scored; ++l) {
+    if (slots[l] < 0 || slots[l] >= n_slots) return cudaErrorInvalidValue;
+    p.layer_of[l] = slots[l];
+  }
+  p.n_slots = n_slots;
   p.ctrl = ws.counters;
   p.status = status;
   p.wait_cycles = wait_limit_cycles();
-  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * g.units, st);
+  cudaError_t e = cudaMemsetAsync(ws.counters, 0, sizeof(int) * 2 * p.units, st);
   if (e != cudaSuccess) return e;
   constexpr int smem = smem_bytes<NR>();
   static_assert(smem <= 227 * 1024, "shared memory budget");
@@ -637,7 +664,7 @@ cudaError_t launch_nr(const LayerGeom &g, const void *q_win, const void *k, cons
   const int grid = p.total_items < sms ? p.total_items : sms;
   // Cooperative launch: every CTA resident at once, which the cross-CTA waits
   // of the schedule rely on.
-  void *args[] = {(void *)&kmap, (void *)&qmap, (void *)&p};
+  void *args[] = {(void *)&lp};
   e = cudaLaunchCooperativeKernel((const void *)score_tc_kernel<NR>, dim3(grid), dim3(kThreads),
                                   args, (size_t)smem, st);
   count_launches(1);
@@ -651,11 +678,19 @@ bool score_tc_supported(const LayerGeom &g) {
          encode_fn() != nullptr;
 }
 
+cudaError_t launch_score_tc(const LayerGeom &g, int n_slots, const int *slots, int n_scored,
+                            const void *const *q_win, const void *const *k, const CompressWs &ws,
+                            float *votes, int32_t *status, cudaStream_t st) {
+  if (g.R == 128)
+    return launch_nr<1>(g, n_slots, slots, n_scored, q_win, k, ws, votes, status, st);
+  return launch_nr<2>(g, n_slots, slots, n_scored, q_win, k, ws, votes, status, st);
+}
+
 cudaError_t launch_score_tc(const LayerGeom &g, const void *q_win, const void *k,
                             const CompressWs &ws, float *votes, int32_t *status,
                             cudaStream_t st) {
-  if (g.R == 128) return launch_nr<1>(g, q_win, k, ws, votes, status, st);
-  return launch_nr<2>(g, q_win, k, ws, votes, status, st);
+  const int slot = 0;
+  return launch_score_tc(g, 1, &slot, 1, &q_win, &k, ws, votes, status, st);
 }
 
 }  // namespace ripple
