@@ -5,8 +5,10 @@
 // causal inside the window, softmax per row over all visible keys, vote of a
 // prefix key = sum over rows of its probability.
 //
-// One launch per layer, one persistent CTA per SM, co-resident (cooperative
-// launch). A unit (b, h) is cut into items of `tpi` key tiles; item i belongs
+// One launch for all the layers of a call (a unit is a (layer, b, h); each
+// layer's keys and queries come through its own tensor maps and its votes go
+// to its slot of the vote array), one persistent CTA per SM, co-resident
+// (cooperative launch). A unit is cut into items of `tpi` key tiles; item i belongs
 // to CTA i mod grid, so every unit is spread over many CTAs that work on it at
 // the same time. Each CTA runs its items in the order
 //     P1(a0) P1(a1) P2(a0) P1(a2) P2(a1) ...
