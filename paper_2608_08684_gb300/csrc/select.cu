@@ -404,10 +404,7 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kCThreads)
     for (int base = 0; base < n_local; base += kCThreads) {
       const int t = base + tid;
       const uint32_t u = t < n_local ? keys[t] : 0u;
-      const bool hit = t < n_local && (u & mask) == prefix;
-      const uint32_t bin = hit ? (u >> shift) & dmask : 0xffffffffu;
-      const uint32_t peers = __match_any_sync(0xffffffffu, bin);
-      if (hit && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
+      if (t < n_local && (u & mask) == prefix) atomicAdd(&hist[(u >> shift) & dmask], 1u);
     }
     cluster_sync_all();  // every CTA's histogram of this round is complete
     // Thread j sums digits 2047-4j .. 2044-4j (descending) over the cluster:
