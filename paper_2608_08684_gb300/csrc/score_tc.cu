@@ -50,7 +50,13 @@ constexpr int kHalfBytes = kTile * 64 * 2;      // 64 bf16 columns of 128 rows: 
 constexpr int kTileBytes = 2 * kHalfBytes;      // one 128 x 128 bf16 tile
 constexpr int kThreads = 352;
 constexpr int kPubSlots = 2;
-constexpr int kMinTilesPerItem = 14;
+// Items of at least 64 key tiles: with every layer of a call in one launch the
+// pipeline's fill and drain no longer favour small items, and fewer items
+// mean fewer partial statistics to publish and merge (80 layers of the 70B
+// shape: 12.36 / 12.07 / 11.76 / 11.59 / 11.58 / 11.53 / 13.11 ms with items
+// of 14 / 18 / 32 / 64 / 128 / 256 / 1024 tiles; one item per unit leaves the
+// last wave of units short).
+constexpr int kMinTilesPerItem = 64;
 
 
 // ------------------------------------------------------------ work list
