@@ -80,6 +80,35 @@ def test_budget_edges(lib, budget):
     assert agree >= 0.999 * total
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_window_only_prompt(lib, dtype):
+    # T = w: no prefix to score (P = 0); every budget keeps the whole window,
+    # in one call and in a multi-layer call
+    wl = synth.WORKLOADS["tiny"].replace(dtype=dtype, head_dim=128 if dtype == "bf16" else 64,
+                                         seq_len=32, window=32, seed=22)
+    q_win, k, v = (t.to(DEV) for t in C.layer_inputs(wl, 0, "cpu"))
+    for budget in (0, 7, 32, 10**6):
+        out = C.run_compress(lib, wl, budget, q_win, k, v, scores=False)
+        assert out["n"] == wl.seq_len
+        assert torch.equal(out["k_out"], k) and torch.equal(out["v_out"], v)
+        assert torch.equal(out["idx"][0, 0].cpu(), torch.arange(wl.seq_len, dtype=torch.int32))
+    B, H, d = wl.batch, wl.n_kv_heads, wl.head_dim
+    desc = lib.layer_desc(B, wl.n_q_heads, H, d, wl.seq_len, wl.window, wl.pool_kernel, "max",
+                          wl.torch_dtype)
+    k_out = [torch.zeros_like(k) for _ in range(2)]
+    v_out = [torch.zeros_like(v) for _ in range(2)]
+    idx = [torch.full((B * H * wl.seq_len,), -1, dtype=torch.int32, device=DEV) for _ in range(2)]
+    tables = lib.CompressTables([q_win] * 2, [k] * 2, [v] * 2, k_out, v_out, idx)
+    ws = torch.empty(lib.ripple_compress_layers_workspace_bytes(desc, 2), dtype=torch.uint8,
+                     device=DEV)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    assert lib.ripple_compress_layers(desc, [3, 500], tables, ws, dev_status=status) == [32, 32]
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    for l in range(2):
+        assert torch.equal(k_out[l], k) and torch.equal(v_out[l], v)
+
+
 def test_keep_all_copies_cache_exactly(lib):
     wl = synth.WORKLOADS["tiny"].replace(dtype="bf16", head_dim=128, seed=21)
     q_win, k, v = (t.to(DEV) for t in C.layer_inputs(wl, 0, "cpu"))
