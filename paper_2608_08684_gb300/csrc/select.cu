@@ -14,7 +14,9 @@
 //   3. an ordered compaction writes every token with key > tau and the first
 //      tokens with key == tau (lower index wins ties) in ascending order,
 //      followed by the w window positions P..T-1.
-// The result is bit-exact and deterministic for a given vote array.
+// The result is bit-exact and deterministic for a given vote array. In a
+// multi-layer call select_unit_kernel also gathers its unit's kept K and V
+// rows (as gather_kernel would), so selection and gather are one launch.
 #include <math.h>
 
 #include "common.cuh"
