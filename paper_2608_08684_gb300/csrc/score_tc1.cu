@@ -524,6 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t id_pv = idesc_bf16(128, 128) | (1u << 15) | (1u << 16);
       const uint32_t kbase = smem_u32(ktiles), qsbase = smem_u32(qsm), q1base = smem_u32(q1m);
       const uint32_t pbase = smem_u32(ptile);
+      const uint64_t q1d = sw128_desc(q1base), qsd = sw128_desc(qsbase);
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
@@ -551,10 +552,14 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
+            // K step kk: 16 keys further along both MN-major operands
+            const uint64_t pd = sw128_desc_mn(pbase, kHalfBytes, 1024);
+            const uint64_t vd = sw128_desc_mn(ka, kHalfBytes, 1024);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              mma_bf16(tmem + C::OCol, sw128_desc_mn(pbase + kk * 2048, kHalfBytes, 1024),
-                       sw128_desc_mn(ka + kk * 2048, kHalfBytes, 1024), id_pv, kk > 0 || s > 0);
+            for (int kk = 0; kk < 8; ++kk) {
+              const uint64_t step = (uint64_t)(kk * 2048 >> 4);
+              mma_bf16(tmem + C::OCol, pd + step, vd + step, id_pv, kk > 0 || s > 0);
+            }
             mma_commit(&ms->k_empty[ks]);
             mma_commit(&ms->p_empty);
             ++kcount;
@@ -580,17 +585,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t d = tmem + as * 128;
-          if (pass == 1) {
+          {
+            // descriptors of the tile's first K step; the others differ only
+            // in their start-address field (16-byte units, no carry)
+            const uint64_t kd = sw128_desc(ka);
+            const uint64_t qd = pass == 1 ? q1d : qsd;
+            const uint64_t ad = pass == 1 ? qd : kd, bd = pass == 1 ? kd : qd;
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) {
-              const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-              mma_bf16(d, sw128_desc(q1base + off), sw128_desc(ka + off), id, kk > 0);
-            }
-          } else {
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-              mma_bf16(d, sw128_desc(ka + off), sw128_desc(qsbase + off), id, kk > 0);
+              const uint64_t off = (uint64_t)(((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4);
+              mma_bf16(d, ad + off, bd + off, id, kk > 0);
             }
           }
           mma_commit(&ms->k_empty[ks]);
