@@ -454,6 +454,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int k = 0; k < n + kLag && ok; ++k) {
         const Step st = step_of(p, k, n);
+        const int l1 = st.u1 / p.upl, loc1 = st.u1 - l1 * p.upl;
+        const int l2 = st.u2 / p.upl, loc2 = st.u2 - l2 * p.upl;
         const int len = kO ? st.n1 + 2 * st.n2 : st.len;
         for (int j = 0; j < len && ok; ++j) {
           int pass, s, kind;
@@ -492,7 +494,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(qsm + kHalfBytes, &lp.qmap[layer], 64, qrow0, &ms->qs_full);
             ++qcount;
           }
-          const int unit = pass == 1 ? st.u1 : st.u2;
           const int tt = pass == 1 ? st.a0 + s : st.b0 + s;
           const int ks = kcount % C::NK;
           if (!wait_bar(&ms->k_empty[ks], ((kcount / C::NK) & 1) ^ 1, ms, p.status)) {
@@ -502,9 +503,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(&ms->k_full[ks], kTileBytes);
           uint8_t *kb = ktiles + ks * kTileBytes;
           const uint64_t pol = pass == 1 ? keep : drop;
-          const CUtensorMap *km =
-              kind == 3 ? &lp.vmap[unit / p.upl] : &lp.kmap[unit / p.upl];
-          const int local = unit % p.upl;
+          // the step's two units' layers and local indices (divisions hoisted
+          // out of the tile loop)
+          const int layer = pass == 1 ? l1 : l2, local = pass == 1 ? loc1 : loc2;
+          const CUtensorMap *km = kind == 3 ? &lp.vmap[layer] : &lp.kmap[layer];
           tma_load_3d(kb, km, 0, tt * kTile, local, &ms->k_full[ks], pol);
           tma_load_3d(kb + kHalfBytes, km, 64, tt * kTile, local, &ms->k_full[ks], pol);
           ++kcount;
